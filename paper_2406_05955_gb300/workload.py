@@ -1,0 +1,156 @@
+"""Seeded synthetic inputs for the sparse dReLU FFN: weights, tokens, routers, predictor lists.
+
+This module draws inputs only; it holds none of the method's arithmetic. The
+CUDA path and the CPU oracle both consume what it returns.
+
+Recipe (shapes and activation rates of the paper's Mistral / Mixtral FFNs,
+Sec. 5 and Sec. 6.2; the real checkpoints and activations are not available):
+
+* Every matrix is neuron-major ``[m][d]``.
+* ``W_gate``, ``W_up`` entries ~ N(0, 1/d); the last input column (index d-1) of
+  both holds one shared per-neuron offset ``b_j ~ N(mu, sigma_b^2)``.
+* ``W_down`` entries ~ N(0, 1/m).
+* Token activations have the bias channel ``x[d-1] = 1`` and unit-variance
+  entries elsewhere, so the pre-activations of neuron j are
+  ``g_j = z_g + b_j``, ``u_j = z_u + b_j`` with ``z ~ N(0, ~1)``. The fraction of
+  gate-active neurons is ``Phi(mu / sqrt(1 + sigma_b^2))`` and of both-active
+  neurons ``E_b[Phi(b)^2]``; ``MU_FOR_ACTIVATION`` solves the latter for mu.
+  The spread of ``b_j`` makes some neurons hot and others cold.
+* bf16 tensors are rounded to nearest-even from the fp32 draw.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass
+
+import torch
+
+# offset mean mu for a target both-active fraction at sigma_b = 0.5
+MU_FOR_ACTIVATION = {0.05: -0.999, 0.10: -0.662, 0.20: -0.250, 0.25: -0.092, 0.50: 0.550}
+# offset for the "every neuron active" case: g, u = N(0,1) + 10 > 0
+ALL_ACTIVE_OFFSET = 10.0
+SIGMA_B = 0.5
+
+
+@dataclass
+class FfnLayer:
+    """One dReLU FFN's weights (``[m][d]`` each) and the offsets written into column d-1."""
+    w_gate: torch.Tensor
+    w_up: torch.Tensor
+    w_down: torch.Tensor
+    offsets: torch.Tensor  # fp32 [m], before rounding to the weight dtype
+
+    @property
+    def d(self) -> int:
+        return int(self.w_gate.shape[1])
+
+    @property
+    def m(self) -> int:
+        return int(self.w_gate.shape[0])
+
+
+def _gen(seed: int, device) -> torch.Generator:
+    g = torch.Generator(device=torch.device(device))
+    g.manual_seed(int(seed))
+    return g
+
+
+def mu_for(activation: float) -> float | None:
+    """Offset mean for a target both-active fraction; None means every neuron active."""
+    if activation >= 1.0:
+        return None
+    return MU_FOR_ACTIVATION[round(float(activation), 2)]
+
+
+def ffn_layer(d: int, m: int, *, activation: float = 0.10, mu: float | None = None,
+              sigma_b: float = SIGMA_B, dtype=torch.bfloat16, seed: int = 0,
+              device="cpu") -> FfnLayer:
+    """Draw one FFN layer. ``mu`` overrides ``activation``; ``activation >= 1`` gives all-active."""
+    g = _gen(seed, device)
+    if mu is None:
+        mu = mu_for(activation)
+    wg = torch.randn(m, d, generator=g, device=device) / math.sqrt(d)
+    wu = torch.randn(m, d, generator=g, device=device) / math.sqrt(d)
+    if mu is None:
+        b = torch.full((m,), ALL_ACTIVE_OFFSET, device=device)
+    else:
+        b = mu + sigma_b * torch.randn(m, generator=g, device=device)
+    wg[:, d - 1] = b
+    wu[:, d - 1] = b
+    wd = torch.randn(m, d, generator=g, device=device) / math.sqrt(m)
+    return FfnLayer(wg.to(dtype).contiguous(), wu.to(dtype).contiguous(),
+                    wd.to(dtype).contiguous(), b.float())
+
+
+def tokens(B: int, d: int, *, dtype=torch.bfloat16, seed: int = 0, device="cpu") -> torch.Tensor:
+    """Token activations ``[B][d]``: N(0,1) entries with the bias channel ``x[:, d-1] = 1``."""
+    x = torch.randn(B, d, generator=_gen(seed, device), device=device)
+    x[:, d - 1] = 1.0
+    return x.to(dtype).contiguous()
+
+
+def residual(B: int, d: int, *, seed: int = 0, device="cpu") -> torch.Tensor:
+    """Initial residual stream ``h_0 [B][d]`` (fp32, N(0,1)) of the synthetic layer stack."""
+    return torch.randn(B, d, generator=_gen(seed, device), device=device).contiguous()
+
+
+def router(E: int, d: int, *, dtype=torch.bfloat16, seed: int = 0, device="cpu") -> torch.Tensor:
+    """Router matrix ``W_r [E][d]`` with N(0, 1/d) entries."""
+    w = torch.randn(E, d, generator=_gen(seed, device), device=device) / math.sqrt(d)
+    return w.to(dtype).contiguous()
+
+
+def predictor_list(offsets: torch.Tensor, k: int, *, zipf_s: float = 1.1, seed: int = 0) -> torch.Tensor:
+    """A predictor's neuron list: k distinct neurons, sorted ascending, int32.
+
+    Neurons are ranked by offset, hottest (largest ``b_j``) first; k ranks are
+    drawn without replacement with Zipf weights ``(r+1)^-s``, so the list
+    favours hot neurons the way a trained predictor would.
+    """
+    b = offsets.detach().float().cpu()
+    m = b.numel()
+    k = max(0, min(int(k), m))
+    if k == 0:
+        return torch.zeros(0, dtype=torch.int32)
+    order = torch.argsort(b, descending=True, stable=True)
+    weights = (torch.arange(m, dtype=torch.float64) + 1.0).pow(-zipf_s)
+    ranks = torch.multinomial(weights, k, replacement=False, generator=_gen(seed, "cpu"))
+    rows = order[ranks]
+    return torch.sort(rows).values.to(torch.int32).contiguous()
+
+
+# ---------------------------------------------------------------------------
+# The five workloads (shapes of the paper's Mistral-7B / Mixtral-47B FFNs)
+# ---------------------------------------------------------------------------
+MISTRAL_D, MISTRAL_M = 4096, 14336
+N_LAYERS = 32
+
+WORKLOADS = {
+    "drelu-ffn-fp32-d512-m1408": dict(
+        d=512, m=1408, dtype="f32", batch=1, n_tokens=16, layers=1, mu=-0.7, seed=0,
+        desc="single dReLU FFN, fp32, 16 decode tokens one at a time"),
+    "mistral7b-ffn-stack-bf16-b1-act10": dict(
+        d=MISTRAL_D, m=MISTRAL_M, dtype="bf16", batch=1, layers=N_LAYERS, activation=0.10, seed=1000,
+        desc="32-layer Mistral-shaped FFN stack, ~10% combined activation, batch 1"),
+    "mistral7b-ffn-stack-bf16-sweep": dict(
+        d=MISTRAL_D, m=MISTRAL_M, dtype="bf16", batches=(1, 4, 16, 64),
+        activations=(0.05, 0.10, 0.25, 0.50, 1.0), layers=N_LAYERS, seed=2000,
+        desc="batch x activation sweep on the Mistral-shaped stack, next to dense cuBLAS"),
+    "mixtral47b-moe-stack-bf16-top2": dict(
+        d=MISTRAL_D, m=MISTRAL_M, dtype="bf16", experts=8, top_k=2, batches=(1, 8), layers=N_LAYERS,
+        activation=0.20, seed=3000,
+        desc="32-layer Mixtral-shaped MoE, 8 experts, top-2, ~20% combined activation per expert"),
+    "mistral7b-ffn-stack-bf16-predictor": dict(
+        d=MISTRAL_D, m=MISTRAL_M, dtype="bf16", batch=1, layers=N_LAYERS, activation=0.10,
+        list_len=1434, zipf_s=1.1, seed=1000,
+        desc="predictor-driven mode: per-layer sorted lists of 1434 neurons (Zipf 1.1 over hotness)"),
+}
+
+
+def torch_dtype(name: str):
+    return {"bf16": torch.bfloat16, "f32": torch.float32}[name]
+
+
+def layer_seed(base: int, layer: int, expert: int = 0) -> int:
+    """Seed of layer ``layer`` (and expert ``expert``) of a workload with base seed ``base``."""
+    return int(base) + 1009 * int(layer) + 17 * int(expert)
