@@ -1,0 +1,438 @@
+"""Benchmark: sparse dReLU FFN decode throughput on the 32-layer Mistral-shaped stack.
+
+One step = one decode token (batch 1) through all 32 FFN layers of the
+pre-norm residual stack (d=4096, m=14336, bf16 weights, ~10% combined dReLU
+activation), replayed from one CUDA graph. Weights (11.3 GB) exceed L2, so no
+flush is needed between steps. Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload stack|predictor|moe] [--batch B]
+
+``--impl reference`` times the fp64 CPU oracle on a bounded sample of the
+same workload (host cores only). Under torchrun with N > 1 every rank runs an
+independent replica on its own GPU (the path has no cross-GPU exchange) and
+``value`` counts the tokens of all ranks over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+METRIC = "sparse-FFN decode tokens/s and achieved HBM GB/s vs needed-bytes roofline"
+UNIT = "tokens/s"
+NOMINAL_HBM_GBS = 7900.0
+
+
+def load_peaks() -> dict:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return {"hbm_gbs": float(j["hbm_gbs"]), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "source": "fallback"}
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (replicas only)
+# ---------------------------------------------------------------------------
+class Dist:
+    def __init__(self, n_gpus: int):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+        if self.world > 1:
+            import torch.distributed as dist
+
+            backend = "nccl" if torch.cuda.is_available() else "gloo"
+            dist.init_process_group(backend=backend)
+            self.pg = dist
+        if n_gpus != self.world and self.world > 1 and self.rank == 0:
+            print(f"warning: --gpus {n_gpus} but WORLD_SIZE {self.world}", file=sys.stderr)
+
+    def barrier(self):
+        if self.pg is not None:
+            if torch.cuda.is_available():
+                self.pg.barrier(device_ids=[self.local])
+            else:
+                self.pg.barrier()
+
+    def max(self, v: float) -> float:
+        if self.pg is None:
+            return v
+        dev = torch.device("cuda", self.local) if torch.cuda.is_available() else torch.device("cpu")
+        t = torch.tensor([v], dtype=torch.float64, device=dev)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg is not None:
+            self.pg.destroy_process_group()
+
+
+# ---------------------------------------------------------------------------
+# clock sampling during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines: list[str] = []
+        self.t = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (FileNotFoundError, OSError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.t.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# workload set-up
+# ---------------------------------------------------------------------------
+def make_stack(ts, wl, dev, batch: int, predictor: bool):
+    cfg = wl.WORKLOADS["mistral7b-ffn-stack-bf16-predictor" if predictor else "mistral7b-ffn-stack-bf16-b1-act10"]
+    d, m, n_layers = cfg["d"], cfg["m"], cfg["layers"]
+    layers, ffns, lists = [], [], []
+    for l in range(n_layers):
+        L = wl.ffn_layer(d, m, activation=cfg["activation"], dtype=torch.bfloat16,
+                         seed=wl.layer_seed(cfg["seed"], l), device=dev)
+        layers.append(L)
+        ffns.append(ts.Ffn(L.w_gate, L.w_up, L.w_down, max_batch=batch))
+        if predictor:
+            lists.append(wl.predictor_list(L.offsets, cfg["list_len"], zipf_s=cfg["zipf_s"],
+                                           seed=wl.layer_seed(cfg["seed"], l) + 7).to(dev))
+    return cfg, layers, ffns, (lists if predictor else None)
+
+
+def needed_bytes_stack(ffns, lists, elem=2) -> dict:
+    """Per-layer algorithmic bytes from the last forward's active sets (union over the batch)."""
+    tot_gate_up, tot_down, per = 0, 0, []
+    for l, f in enumerate(ffns):
+        g, b = f.get_active(-1)
+        n_rows = f.m if lists is None else int(lists[l].numel())
+        gate_kernel = (n_rows + len(g)) * f.d * elem  # gate rows + gathered up rows
+        down_kernel = len(b) * f.d * elem
+        tot_gate_up += gate_kernel
+        tot_down += down_kernel
+        per.append((len(g), len(b)))
+    return {"gate_up": tot_gate_up, "down": tot_down, "per_layer_counts": per}
+
+
+def time_graph(graph, stream, steps: int) -> float:
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record(stream)
+    for _ in range(steps):
+        graph.launch(stream)
+    e.record(stream)
+    e.synchronize()
+    return s.elapsed_time(e) / 1e3
+
+
+def time_kernel_gate_up(ts, ffns, x, stream, lists, reps: int) -> float:
+    """Average duration of one gate+up launch (the dominant kernel), CUDA events on its stream."""
+    for f_i, f in enumerate(ffns):
+        f.gate_up(x, active_idx=None if lists is None else lists[f_i], stream=stream)
+    torch.cuda.synchronize()
+    evs = []
+    for _ in range(reps):
+        for f_i, f in enumerate(ffns):
+            s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            s.record(stream)
+            f.gate_up(x, active_idx=None if lists is None else lists[f_i], stream=stream)
+            e.record(stream)
+            evs.append((s, e))
+    torch.cuda.synchronize()
+    return statistics.mean(s.elapsed_time(e) for s, e in evs) / 1e3
+
+
+def dense_cublas_tokens_per_s(layers, batch, dev, steps=10) -> float:
+    """The same 32-layer stack as a dense ReLU-gated FFN on cuBLAS (torch.matmul), graph-replayed."""
+    d = layers[0].d
+    h = torch.randn(batch, d, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def body():
+        hh = h
+        for L in layers:
+            x = (hh * torch.rsqrt(hh.pow(2).mean(-1, keepdim=True) + 1e-5)).to(torch.bfloat16)
+            g = x @ L.w_gate.t()
+            u = x @ L.w_up.t()
+            c = torch.relu(g) * torch.relu(u)
+            hh = hh + (c @ L.w_down.t()).float()
+        return hh
+
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            body()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        body()
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(steps):
+        g.replay()
+    e.record()
+    e.synchronize()
+    return batch * steps / (s.elapsed_time(e) / 1e3)
+
+
+def cpu_baseline(layers, lists, batch, n_layers_total, budget_s=12.0) -> dict:
+    """The oracle as it stands, on the host cores, over a bounded sample of layers."""
+    import oracle
+
+    host = [(oracle.as_array(L.w_gate), oracle.as_array(L.w_up), oracle.as_array(L.w_down))
+            for L in layers[:2]]
+    hl = None if lists is None else [x.cpu().numpy() for x in lists[:2]]
+    rng = np.random.default_rng(0)
+    h = rng.standard_normal((batch, layers[0].d)).astype(np.float32)
+    done = 0
+    t0 = time.perf_counter()
+    while True:
+        i = done % len(host)
+        x = oracle.rmsnorm(h, oracle.BF16)
+        r = oracle.ffn(x, *host[i], rows=None if hl is None else hl[i])
+        h = (h + r["y"]).astype(np.float32)
+        done += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s or done >= 400:
+            break
+    value = batch * done / n_layers_total / el
+    return {"value": value, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+            "sample": f"{done} layer evaluations (cycling over 2 of the {n_layers_total} layers, batch {batch}) "
+                      f"in {el:.1f} s, scaled to full {n_layers_total}-layer tokens"}
+
+
+# ---------------------------------------------------------------------------
+# arms
+# ---------------------------------------------------------------------------
+def run_ours(args, dist: Dist) -> dict | None:
+    import paper_2406_05955_gb300 as ts
+    from paper_2406_05955_gb300 import workload as wl
+
+    dev = torch.device("cuda", dist.local)
+    torch.cuda.set_device(dev)
+    B = args.batch
+    predictor = args.workload == "predictor"
+    cfg, layers, ffns, lists = make_stack(ts, wl, dev, B, predictor)
+    n_layers = cfg["layers"]
+    h0 = wl.residual(B, cfg["d"], seed=cfg["seed"] - 1, device=dev)
+    h = h0.clone()
+    stream = torch.cuda.Stream(device=dev)
+    graph = ts.Graph.stack(ffns, h, active_idx=lists)
+    for _ in range(args.warmup):
+        graph.launch(stream)
+    torch.cuda.synchronize()
+
+    # timed region: K graph replays, barrier + sync on both sides, clocks sampled
+    clocks = ClockSampler(dist.local)
+    dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    elapsed = time_graph(graph, stream, args.steps)
+    torch.cuda.synchronize()
+    dist.barrier()
+    clk = clocks.stop()
+    t_max = dist.max(elapsed)
+    value = B * args.steps * dist.world / t_max
+
+    # end-to-end through the public API with host buffers (pinned), copies inside the timed region
+    h_host = torch.empty_like(h0, device="cpu").pin_memory()
+    h_host.copy_(h0.cpu())
+    out_host = torch.empty_like(h_host).pin_memory()
+    s_ev, e_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    dist.barrier()
+    torch.cuda.synchronize()
+    s_ev.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(args.steps):
+            h.copy_(h_host, non_blocking=True)
+            graph.launch(stream)
+            out_host.copy_(h, non_blocking=True)
+    e_ev.record(stream)
+    e_ev.synchronize()
+    e2e_t = dist.max(s_ev.elapsed_time(e_ev) / 1e3)
+    e2e = {"value": B * args.steps * dist.world / e2e_t, "unit": UNIT,
+           "h2d_bytes_per_step": h_host.numel() * 4, "d2h_bytes_per_step": out_host.numel() * 4}
+
+    # dominant kernel: gate+up, timed alone per layer
+    x = wl.tokens(B, cfg["d"], dtype=torch.bfloat16, seed=5, device=dev)
+    graph.launch(stream)
+    torch.cuda.synchronize()
+    nb = needed_bytes_stack(ffns, lists)
+    t_gate_up = time_kernel_gate_up(ts, ffns, x, stream, lists, reps=3)
+    nb_x = needed_bytes_stack(ffns, lists)  # active sets of the x used in the kernel timing
+    peaks = load_peaks()
+    gate_up_bytes = nb_x["gate_up"] / n_layers
+    achieved = gate_up_bytes / t_gate_up / 1e9
+    step_s = t_max / args.steps
+    needed_per_token = (nb["gate_up"] + nb["down"]) / B
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": ("mistral7b-ffn-stack-bf16-predictor" if predictor
+                                else "mistral7b-ffn-stack-bf16-b1-act10"),
+                   "d": cfg["d"], "m": cfg["m"], "layers": n_layers, "batch": B,
+                   "activation": cfg["activation"], "weights_gb": round(3 * cfg["d"] * cfg["m"] * 2 * n_layers / 1e9, 2),
+                   "l2": "no flush: the 11.3 GB of weights streamed per step exceed the 129 MB L2",
+                   "parallelism": f"replicas x{dist.world}"},
+        "layers_per_s": value * n_layers / B,
+        "needed_bytes_roofline": {
+            "bytes_per_token": needed_per_token,
+            "achieved_gbs": needed_per_token * B / step_s / 1e9,
+            "frac_of_measured": needed_per_token * B / step_s / 1e9 / peaks["hbm_gbs"],
+            "frac_of_nominal": needed_per_token * B / step_s / 1e9 / NOMINAL_HBM_GBS,
+            "gate_active_per_layer": statistics.mean(c[0] for c in nb["per_layer_counts"]),
+            "both_active_per_layer": statistics.mean(c[1] for c in nb["per_layer_counts"]),
+        },
+        "roofline": {"bound": "hbm", "kernel": "k_gate_up (gate GEMV + gathered up projection)",
+                     "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": achieved / peaks["hbm_gbs"], "peak_source": peaks["source"],
+                     "traffic": None, "bytes_per_launch": gate_up_bytes,
+                     "avg_launch_us": t_gate_up * 1e6},
+        "e2e": e2e,
+        "gpu_launches": 2 * n_layers * args.steps,
+        "clocks": clk,
+    }
+    if not args.no_dense:
+        result["dense_cublas"] = {"value": dense_cublas_tokens_per_s(layers, B, dev), "unit": UNIT,
+                                  "what": "same weights, dense ReLU-gated FFN via torch.matmul (cuBLAS), graph-replayed"}
+    if dist.rank == 0 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(layers, lists, B, n_layers)
+    for f in ffns:
+        f.close()
+    graph.close()
+    return result
+
+
+def run_reference(args, dist: Dist) -> dict | None:
+    """The oracle (fp64, host cores) on a bounded sample per step, same metric and config."""
+    if dist.rank != 0:
+        return None
+    import oracle
+    from paper_2406_05955_gb300 import workload as wl
+
+    oracle.build()
+    predictor = args.workload == "predictor"
+    name = "mistral7b-ffn-stack-bf16-predictor" if predictor else "mistral7b-ffn-stack-bf16-b1-act10"
+    cfg = wl.WORKLOADS[name]
+    B = args.batch
+    L = wl.ffn_layer(cfg["d"], cfg["m"], activation=cfg["activation"], dtype=torch.bfloat16,
+                     seed=wl.layer_seed(cfg["seed"], 0))
+    w = (oracle.as_array(L.w_gate), oracle.as_array(L.w_up), oracle.as_array(L.w_down))
+    rows = wl.predictor_list(L.offsets, cfg["list_len"]).numpy() if predictor else None
+    h = wl.residual(B, cfg["d"], seed=cfg["seed"] - 1).numpy()
+
+    def step():
+        x = oracle.rmsnorm(h, oracle.BF16)
+        return oracle.ffn(x, *w, rows=rows)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    el = time.perf_counter() - t0
+    # one step = one layer of the 32-layer stack for B tokens: tokens/s = B / (32 * t_layer)
+    value = B * args.steps / (el * cfg["layers"])
+    return {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+        "config": {"workload": name, "d": cfg["d"], "m": cfg["m"], "layers": cfg["layers"], "batch": B},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+                         "sample": f"each step: one of the {cfg['layers']} layers (batch {B}), scaled to the full stack"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=["stack", "predictor"], default="stack")
+    ap.add_argument("--batch", type=int, default=1)
+    ap.add_argument("--no-dense", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    dist = Dist(args.gpus)
+    try:
+        if args.impl == "reference":
+            res = run_reference(args, dist)
+        else:
+            from __graft_entry__ import build
+
+            if dist.rank == 0:
+                build()
+            dist.barrier()
+            res = run_ours(args, dist)
+        if res is not None and dist.rank == 0:
+            print(json.dumps(res), flush=True)
+    finally:
+        dist.close()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,185 @@
+/*
+ * ts_ffn.h -- C ABI of libtsffn: the decode-time activation-sparse dReLU FFN
+ * of Turbo Sparse (arXiv 2406.05955) on one GB300 (sm_103a).
+ *
+ * The operation (Eq. 1 in Sec. 2 with the dReLU of Eq. 2 in Sec. 3.2):
+ *     g = x W_gate,  u = x W_up,  c = max(0, g) * max(0, u),  y = c W_down
+ * Only neurons with g_j > 0 cost W_up bytes and only neurons with g_j > 0 and
+ * u_j > 0 ("active", the non-zero activations counted in Sec. 6.2) cost
+ * W_down bytes; the result equals the dense formula.
+ *
+ * Layout. All three weight matrices are neuron-major, [m][d] row-major:
+ * row j of w_gate / w_up is neuron j's input weights (column j of the paper's
+ * d x m matrices), row j of w_down is neuron j's output row (row j of the
+ * paper's m x d W_down). Activations x are [batch][d] in the weight dtype;
+ * outputs y and the residual stream h are [batch][d] fp32. Rows of every
+ * weight matrix must start on 16-byte boundaries (pointer 16-byte aligned
+ * and d * sizeof(element) a multiple of 16).
+ *
+ * Ownership. Weights, x, y, h and index lists are caller-owned device
+ * memory; a handle borrows the weight pointers (they must outlive it) and
+ * owns only its scratch, allocated once by *_create.
+ *
+ * Execution. Every *_forward call is asynchronous on `stream`, performs no
+ * host synchronisation and no allocation, and may be captured in a CUDA
+ * graph. One forward may be in flight per handle at a time.
+ *
+ * Errors. Argument errors are returned synchronously and nothing is
+ * launched. Errors the GPU detects (an out-of-range or unsorted index list)
+ * never trap: the offending entries are skipped, a status word in the
+ * handle's scratch records it, and ts_*_get_error reports it.
+ */
+#ifndef TS_FFN_H
+#define TS_FFN_H
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    TS_OK = 0,
+    TS_ERR_INVALID_ARG = 1,  /* bad pointer, size, alignment or batch       */
+    TS_ERR_CUDA = 2,         /* a CUDA runtime call failed                   */
+    TS_ERR_OOM = 3,          /* scratch allocation failed                    */
+    TS_ERR_BAD_INDEX = 4,    /* the GPU saw an out-of-range/unsorted list    */
+    TS_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up           */
+    TS_ERR_UNSUPPORTED = 6   /* valid request this build does not handle     */
+} ts_status;
+
+typedef enum { TS_F32 = 0, TS_BF16 = 1 } ts_dtype;
+
+typedef struct ts_ffn ts_ffn;     /* one dReLU FFN (one layer or one expert) */
+typedef struct ts_moe ts_moe;     /* one top-k MoE layer over ts_ffn experts */
+typedef struct ts_graph ts_graph; /* a captured multi-layer forward          */
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char* ts_status_str(ts_status s);
+
+/* ABI version of this library (major * 100 + minor). */
+int ts_version(void);
+
+/*
+ * Create a handle for one dReLU FFN (Eq. 1 + Eq. 2).
+ *   d, m       model width and number of neurons (d >= 1, m >= 1)
+ *   wdtype     storage type of weights and activations
+ *   w_gate, w_up, w_down  device pointers, [m][d] each (borrowed)
+ *   max_batch  largest batch a forward may pass (1..64)
+ * Allocates the handle's scratch on the current device.
+ * Returns TS_ERR_INVALID_ARG for bad sizes/pointers/alignment, TS_ERR_OOM if
+ * scratch cannot be allocated, TS_ERR_CUDA for other CUDA failures.
+ */
+ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void* w_gate,
+                        const void* w_up, const void* w_down, int max_batch);
+void ts_ffn_destroy(ts_ffn* h);
+
+/*
+ * y = dReLU-FFN(x) for `batch` tokens (Eq. 1 + Eq. 2), on `stream`.
+ *   x          device [batch][d], wdtype
+ *   y          device [batch][d] fp32, overwritten
+ *   active_idx NULL: the active sets are detected from the signs of g and u.
+ *              Otherwise a device list of n_active neuron ids (0 <= n_active
+ *              <= m), strictly ascending, shared by every token of the
+ *              batch: the predictor-driven mode of Sec. 7. Gate, up and
+ *              down then touch only listed rows, and listed neurons that
+ *              are not dReLU-active contribute 0; unlisted neurons are
+ *              skipped even if they would be active.
+ * batch == 0 is a no-op. Equivalent to ts_ffn_gate_up then ts_ffn_down.
+ */
+ts_status ts_ffn_forward(ts_ffn* h, const void* x, int batch, float* y, cudaStream_t stream,
+                         const int32_t* active_idx, int n_active);
+
+/*
+ * First step alone: gate GEMV + ReLU + compaction, then the gathered up
+ * projection over gate-active rows + dReLU product + second compaction
+ * (into the handle's scratch). Arguments as ts_ffn_forward. For batch > 8
+ * the steps run in passes of 8 tokens and ts_ffn_forward must be used.
+ */
+ts_status ts_ffn_gate_up(ts_ffn* h, const void* x, int batch, cudaStream_t stream,
+                         const int32_t* active_idx, int n_active);
+
+/* Second step alone: gathered down projection of the rows the preceding
+   ts_ffn_gate_up on this handle marked active; writes y [batch][d] fp32. */
+ts_status ts_ffn_down(ts_ffn* h, int batch, float* y, cudaStream_t stream);
+
+/*
+ * Pre-norm residual stack of n_layers FFNs on the fp32 residual h [batch][d]
+ * (updated in place): for each layer l,
+ *     x = round_wdtype(h / sqrt(mean(h^2) + 1e-5)),  x[d-1] = 1,
+ *     h = h + FFN_l(x).
+ * (The normalisation and bias channel are synthetic glue: the paper studies
+ * the FFN alone.) active_idx / n_active: NULL, or per-layer lists as in
+ * ts_ffn_forward (an entry may be NULL). All layers need the same d, wdtype.
+ */
+ts_status ts_stack_forward(ts_ffn* const* layers, int n_layers, float* h, int batch,
+                           cudaStream_t stream, const int32_t* const* active_idx,
+                           const int* n_active);
+
+/*
+ * Active sets of the last forward on this handle, copied to host memory
+ * (synchronises `stream`). token >= 0 selects one token, -1 the union over
+ * the batch. gate_idx / both_idx are host arrays of at least m entries
+ * (either may be NULL); the lists come back ascending (neuron ids).
+ */
+ts_status ts_ffn_get_active(ts_ffn* h, cudaStream_t stream, int token, int32_t* gate_idx,
+                            int* n_gate, int32_t* both_idx, int* n_both);
+
+/* Synchronise `stream`, return and clear the device status word:
+   TS_OK or TS_ERR_BAD_INDEX. */
+ts_status ts_ffn_get_error(ts_ffn* h, cudaStream_t stream);
+
+/*
+ * Top-k MoE layer (Sec. 4; Mixtral: 2 of 8 experts, Sec. 6.2):
+ *     r = x W_r^T, pick the top_k largest logits (lower expert index wins a
+ *     tie), w = softmax over the picked logits,
+ *     y_t = sum_k w_{t,k} * FFN_{e_{t,k}}(x_t),
+ * each expert itself a neuron-sparse dReLU FFN.
+ *   w_router   device [n_experts][d], wdtype (borrowed)
+ *   experts    n_experts handles (same d and wdtype; borrowed)
+ *   n_experts  1..16, top_k 1..min(4, n_experts), max_batch 1..8
+ */
+ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype wdtype,
+                        const void* w_router, ts_ffn* const* experts, int max_batch);
+void ts_moe_destroy(ts_moe* h);
+
+/* y [batch][d] fp32 = MoE(x [batch][d] wdtype), on `stream`. */
+ts_status ts_moe_forward(ts_moe* h, const void* x, int batch, float* y, cudaStream_t stream);
+
+/* Pre-norm residual stack of MoE layers on h [batch][d] fp32 (in place),
+   with the same glue as ts_stack_forward. */
+ts_status ts_moe_stack_forward(ts_moe* const* layers, int n_layers, float* h, int batch,
+                               cudaStream_t stream);
+
+/* Routing of the last forward, to host memory (synchronises `stream`):
+   sel [batch][top_k] expert ids (largest logit first), w [batch][top_k]. */
+ts_status ts_moe_get_routing(ts_moe* h, cudaStream_t stream, int32_t* sel, float* w);
+
+/* Per-expert active sets of the last MoE forward (synchronises `stream`):
+   as ts_ffn_get_active for expert `expert` and batch token `token` (-1: the
+   union over the tokens routed to that expert). */
+ts_status ts_moe_get_active(ts_moe* h, cudaStream_t stream, int expert, int token,
+                            int32_t* gate_idx, int* n_gate, int32_t* both_idx, int* n_both);
+
+/* As ts_ffn_get_error, for the MoE layer's router and grouped kernels. */
+ts_status ts_moe_get_error(ts_moe* h, cudaStream_t stream);
+
+/*
+ * Capture a whole multi-layer forward once as a CUDA graph and replay it.
+ * The captured calls keep the pointers given here; replaying reads and
+ * writes the same buffers. ts_graph_capture_stack captures
+ * ts_stack_forward(layers, n_layers, h, batch, ., active_idx, n_active);
+ * ts_graph_capture_moe_stack captures ts_moe_stack_forward.
+ */
+ts_status ts_graph_capture_stack(ts_graph** out, ts_ffn* const* layers, int n_layers, float* h,
+                                 int batch, const int32_t* const* active_idx, const int* n_active);
+ts_status ts_graph_capture_moe_stack(ts_graph** out, ts_moe* const* layers, int n_layers,
+                                     float* h, int batch);
+ts_status ts_graph_launch(ts_graph* g, cudaStream_t stream);
+void ts_graph_destroy(ts_graph* g);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TS_FFN_H */

@@ -1,0 +1,697 @@
+// ts_api.cu -- the C ABI of libtsffn (declared in include/ts_ffn.h): handles,
+// scratch arenas, argument validation, pass splitting, launch sequencing
+// with programmatic dependent launch, active-set export and graph capture.
+#include <stdint.h>
+#include <string.h>
+
+#include <algorithm>
+#include <new>
+#include <vector>
+
+#include "ts_ffn.h"
+#include "ts_kernels.cuh"
+
+using namespace tsffn;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+int elem_size(ts_dtype dt) { return dt == TS_BF16 ? 2 : 4; }
+int pow2_tokens(int nt) { return nt <= 1 ? 1 : nt <= 2 ? 2 : nt <= 4 ? 4 : 8; }
+
+// Device facts needed to size grids; looked up at handle creation.
+struct DeviceInfo {
+    int device = 0;
+    int num_sms = 1;
+    int optin_smem = 48 * 1024;
+};
+
+ts_status device_info(DeviceInfo* di) {
+    if (cudaGetDevice(&di->device) != cudaSuccess) return TS_ERR_CUDA;
+    if (cudaDeviceGetAttribute(&di->num_sms, cudaDevAttrMultiProcessorCount, di->device) != cudaSuccess)
+        return TS_ERR_CUDA;
+    if (cudaDeviceGetAttribute(&di->optin_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, di->device) !=
+        cudaSuccess)
+        return TS_ERR_CUDA;
+    if (prepare_gate_up(di->optin_smem) != cudaSuccess || prepare_down() != cudaSuccess ||
+        prepare_router() != cudaSuccess)
+        return TS_ERR_CUDA;
+    return TS_OK;
+}
+
+// Carves sub-buffers out of one device allocation.
+struct Arena {
+    size_t bytes = 0;
+    char* base = nullptr;
+    size_t take(size_t n) {
+        const size_t off = bytes;
+        bytes += align_up(n);
+        return off;
+    }
+    template <typename P>
+    P* at(size_t off) const { return reinterpret_cast<P*>(base + off); }
+};
+
+ts_status alloc_arena(Arena* ar) {
+    if (cudaMalloc(&ar->base, ar->bytes) != cudaSuccess) {
+        cudaGetLastError();
+        ar->base = nullptr;
+        return TS_ERR_OOM;
+    }
+    if (cudaMemset(ar->base, 0, ar->bytes) != cudaSuccess) {
+        cudaFree(ar->base);
+        ar->base = nullptr;
+        return TS_ERR_CUDA;
+    }
+    return TS_OK;
+}
+
+// Scratch of the grouped kernels: per-expert c values and bitmaps, the down
+// projection's partials and tickets, and the device status word.
+struct Scratch {
+    float* cval = nullptr;
+    uint8_t* gbits = nullptr;
+    uint8_t* bbits = nullptr;
+    uint8_t* ubits = nullptr;
+    uint8_t* ugbits = nullptr;
+    float* partial = nullptr;
+    unsigned* counters = nullptr;
+    unsigned* status = nullptr;
+};
+
+int down_col_slices(int d) { return (d + kColSlice - 1) / kColSlice; }
+int down_row_groups(int d, int num_sms) { return std::max(1, 2 * num_sms / down_col_slices(d)); }
+
+}  // namespace
+
+struct ts_ffn {
+    int d = 0, m = 0, max_batch = 0;
+    ts_dtype dt = TS_BF16;
+    const void* wg = nullptr;
+    const void* wu = nullptr;
+    const void* wd = nullptr;
+    DeviceInfo dev;
+    int n_cs = 0, n_rg = 0, nbytes = 0;
+    Arena arena;
+    Scratch s;
+    int grid[9] = {0};  // gate+up grid per pass width 1, 2, 4, 8
+    // the last gate+up on this handle (read by ts_ffn_down and the exports)
+    int last_batch = 0;
+    const int32_t* last_rows = nullptr;
+    int last_n_rows = 0;
+};
+
+struct ts_moe {
+    int d = 0, m = 0, E = 0, top_k = 0, max_batch = 0;
+    ts_dtype dt = TS_BF16;
+    const void* wr = nullptr;
+    ExpertPtrs ex[kMaxExperts];
+    DeviceInfo dev;
+    int n_cs = 0, n_rg = 0, nbytes = 0;
+    Arena arena;
+    Scratch s;
+    TokenRoute* route = nullptr;
+    void* xbuf = nullptr;
+    int grid[9] = {0};
+    int last_batch = 0;
+};
+
+struct ts_graph {
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+};
+
+extern "C" {
+
+const char* ts_status_str(ts_status s) {
+    switch (s) {
+        case TS_OK: return "TS_OK";
+        case TS_ERR_INVALID_ARG: return "TS_ERR_INVALID_ARG";
+        case TS_ERR_CUDA: return "TS_ERR_CUDA";
+        case TS_ERR_OOM: return "TS_ERR_OOM";
+        case TS_ERR_BAD_INDEX: return "TS_ERR_BAD_INDEX";
+        case TS_ERR_TIMEOUT: return "TS_ERR_TIMEOUT";
+        case TS_ERR_UNSUPPORTED: return "TS_ERR_UNSUPPORTED";
+    }
+    return "TS_ERR_UNKNOWN";
+}
+
+int ts_version(void) { return 100; }
+
+ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void* w_gate,
+                        const void* w_up, const void* w_down, int max_batch) {
+    if (out == nullptr) return TS_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (d < 1 || m < 1 || max_batch < 1 || max_batch > kMaxBatch) return TS_ERR_INVALID_ARG;
+    if (wdtype != TS_F32 && wdtype != TS_BF16) return TS_ERR_INVALID_ARG;
+    if (!w_gate || !w_up || !w_down) return TS_ERR_INVALID_ARG;
+    if (!aligned16(w_gate) || !aligned16(w_up) || !aligned16(w_down)) return TS_ERR_INVALID_ARG;
+    if (((size_t)d * elem_size(wdtype)) % 16 != 0) return TS_ERR_INVALID_ARG;
+    if (m > (1 << 28) || (size_t)d * (size_t)m > ((size_t)1 << 40)) return TS_ERR_UNSUPPORTED;
+
+    DeviceInfo dev;
+    ts_status st = device_info(&dev);
+    if (st != TS_OK) return st;
+    const int pass_cap = std::min(max_batch, kMaxPass);
+    if ((size_t)pass_cap * d * sizeof(float) + 4096 > (size_t)dev.optin_smem) return TS_ERR_UNSUPPORTED;
+
+    ts_ffn* h = new (std::nothrow) ts_ffn();
+    if (!h) return TS_ERR_OOM;
+    h->d = d;
+    h->m = m;
+    h->max_batch = max_batch;
+    h->dt = wdtype;
+    h->wg = w_gate;
+    h->wu = w_up;
+    h->wd = w_down;
+    h->dev = dev;
+    h->n_cs = down_col_slices(d);
+    h->n_rg = down_row_groups(d, dev.num_sms);
+    h->nbytes = (m + 31) / 32 * 4;
+    const size_t o_cval = h->arena.take((size_t)kMaxPass * m * sizeof(float));
+    const size_t o_g = h->arena.take((size_t)max_batch * h->nbytes);
+    const size_t o_b = h->arena.take((size_t)max_batch * h->nbytes);
+    const size_t o_u = h->arena.take((size_t)h->nbytes);
+    const size_t o_ug = h->arena.take((size_t)h->nbytes);
+    const size_t o_p = h->arena.take((size_t)h->n_rg * kMaxPass * d * sizeof(float));
+    const size_t o_c = h->arena.take((size_t)h->n_cs * sizeof(unsigned));
+    const size_t o_s = h->arena.take(sizeof(unsigned));
+    st = alloc_arena(&h->arena);
+    if (st != TS_OK) {
+        delete h;
+        return st;
+    }
+    h->s.cval = h->arena.at<float>(o_cval);
+    h->s.gbits = h->arena.at<uint8_t>(o_g);
+    h->s.bbits = h->arena.at<uint8_t>(o_b);
+    h->s.ubits = h->arena.at<uint8_t>(o_u);
+    h->s.ugbits = h->arena.at<uint8_t>(o_ug);
+    h->s.partial = h->arena.at<float>(o_p);
+    h->s.counters = h->arena.at<unsigned>(o_c);
+    h->s.status = h->arena.at<unsigned>(o_s);
+    const int n_chunks = (m + kChunk - 1) / kChunk;
+    for (int nt : {1, 2, 4, 8}) {
+        const int per_sm = gate_up_blocks_per_sm(wdtype, nt, nt, d);
+        const int need = (n_chunks + kGateUpWarps - 1) / kGateUpWarps;
+        h->grid[nt] = std::max(1, std::min(per_sm * dev.num_sms, need));
+    }
+    *out = h;
+    return TS_OK;
+}
+
+void ts_ffn_destroy(ts_ffn* h) {
+    if (!h) return;
+    if (h->arena.base) cudaFree(h->arena.base);
+    delete h;
+}
+
+}  // extern "C"
+
+namespace {
+
+FfnLaunch ffn_launch(const ts_ffn* h, int batch, const int32_t* rows, int n_rows) {
+    FfnLaunch a;
+    memset(&a, 0, sizeof a);
+    a.d = h->d;
+    a.m = h->m;
+    a.rows = rows;
+    a.n_rows = rows ? n_rows : h->m;
+    a.batch = batch;
+    a.n_experts = 1;
+    a.ex[0] = ExpertPtrs{h->wg, h->wu, h->wd};
+    a.route = nullptr;
+    a.top_k = 1;
+    a.cval = h->s.cval;
+    a.cval_tok_stride = h->m;
+    a.gbits = h->s.gbits;
+    a.bbits = h->s.bbits;
+    a.bits_expert_stride = 0;
+    a.nbytes = h->nbytes;
+    a.ubits = h->s.ubits;
+    a.ugbits = h->s.ugbits;
+    a.partial = h->s.partial;
+    a.counters = h->s.counters;
+    a.status = h->s.status;
+    a.n_rg = h->n_rg;
+    a.n_cs = h->n_cs;
+    return a;
+}
+
+ts_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TS_OK : TS_ERR_CUDA; }
+
+ts_status check_list(const ts_ffn* h, const int32_t* idx, int n) {
+    if (idx != nullptr && (n < 0 || n > h->m)) return TS_ERR_INVALID_ARG;
+    return TS_OK;
+}
+
+// gate+up (and down) for tokens tok0 .. tok0+nt-1 of the call.
+ts_status run_pass(ts_ffn* h, FfnLaunch a, int tok0, int nt, cudaStream_t stream, bool gate_up,
+                   bool down) {
+    a.tok0 = tok0;
+    a.nt = nt;
+    a.bits_tok_base = tok0;
+    const int w = pow2_tokens(nt);
+    if (gate_up) {
+        ts_status st = cuda_status(launch_gate_up(a, h->dt, w, h->grid[w], stream, true));
+        if (st != TS_OK) return st;
+    }
+    if (down) return cuda_status(launch_down(a, h->dt, w, stream, true));
+    return TS_OK;
+}
+
+void remember(ts_ffn* h, int batch, const int32_t* rows, int n_rows) {
+    h->last_batch = batch;
+    h->last_rows = rows;
+    h->last_n_rows = rows ? n_rows : h->m;
+}
+
+// Decode bitmap bytes of the row space into ascending neuron ids.
+int decode_bits(const uint8_t* bits, int n_rows, const std::vector<int32_t>& rows, int32_t* out) {
+    int n = 0;
+    for (int p = 0; p < n_rows; ++p)
+        if ((bits[p >> 3] >> (p & 7)) & 1u) {
+            if (out) out[n] = rows.empty() ? p : rows[p];
+            ++n;
+        }
+    return n;
+}
+
+// Host copies of per-token bitmaps (token >= 0) or their union over `tokens`.
+ts_status fetch_active(cudaStream_t stream, const uint8_t* gbits_dev, const uint8_t* bbits_dev,
+                       int nbytes, int n_rows, const int32_t* rows_dev, int token_first,
+                       int n_tokens, int32_t* gate_idx, int* n_gate, int32_t* both_idx, int* n_both) {
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return TS_ERR_CUDA;
+    std::vector<uint8_t> g((size_t)n_tokens * nbytes), b((size_t)n_tokens * nbytes);
+    if (n_tokens > 0) {
+        if (cudaMemcpy(g.data(), gbits_dev + (size_t)token_first * nbytes, g.size(),
+                       cudaMemcpyDeviceToHost) != cudaSuccess ||
+            cudaMemcpy(b.data(), bbits_dev + (size_t)token_first * nbytes, b.size(),
+                       cudaMemcpyDeviceToHost) != cudaSuccess)
+            return TS_ERR_CUDA;
+    }
+    std::vector<uint8_t> gu(nbytes, 0), bu(nbytes, 0);
+    for (int t = 0; t < n_tokens; ++t)
+        for (int i = 0; i < nbytes; ++i) {
+            gu[i] |= g[(size_t)t * nbytes + i];
+            bu[i] |= b[(size_t)t * nbytes + i];
+        }
+    std::vector<int32_t> rows;
+    if (rows_dev != nullptr && n_rows > 0) {
+        rows.resize(n_rows);
+        if (cudaMemcpy(rows.data(), rows_dev, n_rows * sizeof(int32_t), cudaMemcpyDeviceToHost) !=
+            cudaSuccess)
+            return TS_ERR_CUDA;
+    }
+    const int ng = decode_bits(gu.data(), n_rows, rows, gate_idx);
+    const int nb = decode_bits(bu.data(), n_rows, rows, both_idx);
+    if (n_gate) *n_gate = ng;
+    if (n_both) *n_both = nb;
+    return TS_OK;
+}
+
+ts_status read_status(unsigned* status_dev, cudaStream_t stream) {
+    unsigned v = 0;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return TS_ERR_CUDA;
+    if (cudaMemcpy(&v, status_dev, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return TS_ERR_CUDA;
+    if (cudaMemset(status_dev, 0, sizeof v) != cudaSuccess) return TS_ERR_CUDA;
+    return (v & kStatusBadIndex) ? TS_ERR_BAD_INDEX : TS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+ts_status ts_ffn_forward(ts_ffn* h, const void* x, int batch, float* y, cudaStream_t stream,
+                         const int32_t* active_idx, int n_active) {
+    if (!h || batch < 0 || batch > h->max_batch) return TS_ERR_INVALID_ARG;
+    if (batch == 0) return TS_OK;
+    if (!x || !y) return TS_ERR_INVALID_ARG;
+    ts_status st = check_list(h, active_idx, n_active);
+    if (st != TS_OK) return st;
+    FfnLaunch a = ffn_launch(h, batch, active_idx, n_active);
+    a.x = x;
+    a.y = y;
+    for (int t0 = 0; t0 < batch; t0 += kMaxPass) {
+        st = run_pass(h, a, t0, std::min(kMaxPass, batch - t0), stream, true, true);
+        if (st != TS_OK) return st;
+    }
+    remember(h, batch, active_idx, n_active);
+    return TS_OK;
+}
+
+ts_status ts_ffn_gate_up(ts_ffn* h, const void* x, int batch, cudaStream_t stream,
+                         const int32_t* active_idx, int n_active) {
+    if (!h || batch < 0 || batch > h->max_batch) return TS_ERR_INVALID_ARG;
+    if (batch > kMaxPass) return TS_ERR_UNSUPPORTED;
+    if (batch == 0) return TS_OK;
+    if (!x) return TS_ERR_INVALID_ARG;
+    ts_status st = check_list(h, active_idx, n_active);
+    if (st != TS_OK) return st;
+    FfnLaunch a = ffn_launch(h, batch, active_idx, n_active);
+    a.x = x;
+    st = run_pass(h, a, 0, batch, stream, true, false);
+    if (st == TS_OK) remember(h, batch, active_idx, n_active);
+    return st;
+}
+
+ts_status ts_ffn_down(ts_ffn* h, int batch, float* y, cudaStream_t stream) {
+    if (!h || batch < 0 || batch > kMaxPass) return TS_ERR_INVALID_ARG;
+    if (batch == 0) return TS_OK;
+    if (!y || batch != h->last_batch) return TS_ERR_INVALID_ARG;
+    FfnLaunch a = ffn_launch(h, batch, h->last_rows, h->last_n_rows);
+    a.y = y;
+    return run_pass(h, a, 0, batch, stream, false, true);
+}
+
+ts_status ts_stack_forward(ts_ffn* const* layers, int n_layers, float* hres, int batch,
+                           cudaStream_t stream, const int32_t* const* active_idx,
+                           const int* n_active) {
+    if (!layers || n_layers < 0 || !hres || batch < 0) return TS_ERR_INVALID_ARG;
+    if (batch == 0 || n_layers == 0) return TS_OK;
+    for (int l = 0; l < n_layers; ++l) {
+        const ts_ffn* h = layers[l];
+        if (!h || h->d != layers[0]->d || h->dt != layers[0]->dt || batch > h->max_batch)
+            return TS_ERR_INVALID_ARG;
+        const int32_t* rows = active_idx ? active_idx[l] : nullptr;
+        if (rows && !n_active) return TS_ERR_INVALID_ARG;
+        ts_status st = check_list(h, rows, rows ? n_active[l] : 0);
+        if (st != TS_OK) return st;
+    }
+    for (int l = 0; l < n_layers; ++l) {
+        ts_ffn* h = layers[l];
+        const int32_t* rows = active_idx ? active_idx[l] : nullptr;
+        const int nr = rows ? n_active[l] : 0;
+        FfnLaunch a = ffn_launch(h, batch, rows, nr);
+        a.h = hres;
+        a.norm_from_h = 1;
+        a.residual_out = 1;
+        for (int t0 = 0; t0 < batch; t0 += kMaxPass) {
+            ts_status st = run_pass(h, a, t0, std::min(kMaxPass, batch - t0), stream, true, true);
+            if (st != TS_OK) return st;
+        }
+        remember(h, batch, rows, nr);
+    }
+    return TS_OK;
+}
+
+ts_status ts_ffn_get_active(ts_ffn* h, cudaStream_t stream, int token, int32_t* gate_idx,
+                            int* n_gate, int32_t* both_idx, int* n_both) {
+    if (!h || token < -1 || token >= std::max(h->last_batch, 0)) return TS_ERR_INVALID_ARG;
+    if (h->last_batch == 0) return TS_ERR_INVALID_ARG;
+    const int first = token < 0 ? 0 : token;
+    const int n = token < 0 ? h->last_batch : 1;
+    return fetch_active(stream, h->s.gbits, h->s.bbits, h->nbytes, h->last_n_rows, h->last_rows,
+                        first, n, gate_idx, n_gate, both_idx, n_both);
+}
+
+ts_status ts_ffn_get_error(ts_ffn* h, cudaStream_t stream) {
+    if (!h) return TS_ERR_INVALID_ARG;
+    return read_status(h->s.status, stream);
+}
+
+// ---------------------------------------------------------------------------
+// MoE
+// ---------------------------------------------------------------------------
+ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype wdtype,
+                        const void* w_router, ts_ffn* const* experts, int max_batch) {
+    if (out == nullptr) return TS_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (d < 1 || n_experts < 1 || n_experts > kMaxExperts) return TS_ERR_INVALID_ARG;
+    if (top_k < 1 || top_k > std::min(kMaxTopK, n_experts)) return TS_ERR_INVALID_ARG;
+    if (max_batch < 1 || max_batch > kMaxMoeBatch) return TS_ERR_INVALID_ARG;
+    if (wdtype != TS_F32 && wdtype != TS_BF16) return TS_ERR_INVALID_ARG;
+    if (!w_router || !aligned16(w_router) || !experts) return TS_ERR_INVALID_ARG;
+    if (d > kRouterMaxD) return TS_ERR_UNSUPPORTED;
+    for (int e = 0; e < n_experts; ++e) {
+        const ts_ffn* x = experts[e];
+        if (!x || x->d != d || x->dt != wdtype || x->m != experts[0]->m) return TS_ERR_INVALID_ARG;
+    }
+    DeviceInfo dev;
+    ts_status st = device_info(&dev);
+    if (st != TS_OK) return st;
+    if ((size_t)max_batch * d * sizeof(float) + 4096 > (size_t)dev.optin_smem) return TS_ERR_UNSUPPORTED;
+
+    ts_moe* h = new (std::nothrow) ts_moe();
+    if (!h) return TS_ERR_OOM;
+    h->d = d;
+    h->m = experts[0]->m;
+    h->E = n_experts;
+    h->top_k = top_k;
+    h->max_batch = max_batch;
+    h->dt = wdtype;
+    h->wr = w_router;
+    for (int e = 0; e < n_experts; ++e) h->ex[e] = ExpertPtrs{experts[e]->wg, experts[e]->wu, experts[e]->wd};
+    h->dev = dev;
+    h->n_cs = down_col_slices(d);
+    h->n_rg = down_row_groups(d, dev.num_sms);
+    h->nbytes = (h->m + 31) / 32 * 4;
+    const int m = h->m, E = n_experts;
+    const size_t o_cval = h->arena.take((size_t)E * kMaxPass * m * sizeof(float));
+    const size_t o_g = h->arena.take((size_t)E * kMaxPass * h->nbytes);
+    const size_t o_b = h->arena.take((size_t)E * kMaxPass * h->nbytes);
+    const size_t o_u = h->arena.take((size_t)E * h->nbytes);
+    const size_t o_ug = h->arena.take((size_t)E * h->nbytes);
+    const size_t o_p = h->arena.take((size_t)h->n_rg * kMaxPass * d * sizeof(float));
+    const size_t o_c = h->arena.take((size_t)h->n_cs * sizeof(unsigned));
+    const size_t o_s = h->arena.take(sizeof(unsigned));
+    const size_t o_r = h->arena.take((size_t)max_batch * sizeof(TokenRoute));
+    const size_t o_x = h->arena.take((size_t)max_batch * d * elem_size(wdtype));
+    st = alloc_arena(&h->arena);
+    if (st != TS_OK) {
+        delete h;
+        return st;
+    }
+    h->s.cval = h->arena.at<float>(o_cval);
+    h->s.gbits = h->arena.at<uint8_t>(o_g);
+    h->s.bbits = h->arena.at<uint8_t>(o_b);
+    h->s.ubits = h->arena.at<uint8_t>(o_u);
+    h->s.ugbits = h->arena.at<uint8_t>(o_ug);
+    h->s.partial = h->arena.at<float>(o_p);
+    h->s.counters = h->arena.at<unsigned>(o_c);
+    h->s.status = h->arena.at<unsigned>(o_s);
+    h->route = h->arena.at<TokenRoute>(o_r);
+    h->xbuf = h->arena.at<void>(o_x);
+    const int n_chunks = (m + kChunk - 1) / kChunk;
+    for (int nt : {1, 2, 4, 8}) {
+        const int x_tokens = std::min(nt, max_batch);
+        const int per_sm = gate_up_blocks_per_sm(wdtype, nt, x_tokens, d);
+        const int need = (std::min(E, nt * top_k) * n_chunks + kGateUpWarps - 1) / kGateUpWarps;
+        h->grid[nt] = std::max(1, std::min(per_sm * dev.num_sms, need));
+    }
+    *out = h;
+    return TS_OK;
+}
+
+void ts_moe_destroy(ts_moe* h) {
+    if (!h) return;
+    if (h->arena.base) cudaFree(h->arena.base);
+    delete h;
+}
+
+}  // extern "C"
+
+namespace {
+
+// router -> grouped gate+up -> grouped down for one MoE layer.
+ts_status moe_layer(ts_moe* h, const void* x, float* hres, int batch, float* y, cudaStream_t stream) {
+    RouterLaunch r;
+    memset(&r, 0, sizeof r);
+    r.d = h->d;
+    r.n_experts = h->E;
+    r.top_k = h->top_k;
+    r.batch = batch;
+    r.x = hres ? nullptr : x;
+    r.h = hres;
+    r.xbuf = h->xbuf;
+    r.wr = h->wr;
+    r.route = h->route;
+    ts_status st = cuda_status(launch_router(r, h->dt, stream, true));
+    if (st != TS_OK) return st;
+
+    FfnLaunch a;
+    memset(&a, 0, sizeof a);
+    a.d = h->d;
+    a.m = h->m;
+    a.n_rows = h->m;
+    a.rows = nullptr;
+    a.batch = batch;
+    a.tok0 = 0;
+    a.nt = batch;
+    a.x = hres ? h->xbuf : x;
+    a.h = hres;
+    a.y = y;
+    a.norm_from_h = 0;
+    a.residual_out = hres ? 1 : 0;
+    a.n_experts = h->E;
+    for (int e = 0; e < h->E; ++e) a.ex[e] = h->ex[e];
+    a.route = h->route;
+    a.top_k = h->top_k;
+    a.cval = h->s.cval;
+    a.cval_tok_stride = h->m;
+    a.gbits = h->s.gbits;
+    a.bbits = h->s.bbits;
+    a.bits_expert_stride = (long long)kMaxPass * h->nbytes;
+    a.bits_tok_base = 0;
+    a.nbytes = h->nbytes;
+    a.ubits = h->s.ubits;
+    a.ugbits = h->s.ugbits;
+    a.partial = h->s.partial;
+    a.counters = h->s.counters;
+    a.status = h->s.status;
+    a.n_rg = h->n_rg;
+    a.n_cs = h->n_cs;
+    const int w = pow2_tokens(batch);
+    st = cuda_status(launch_gate_up(a, h->dt, w, h->grid[w], stream, true));
+    if (st != TS_OK) return st;
+    return cuda_status(launch_down(a, h->dt, w, stream, true));
+}
+
+}  // namespace
+
+extern "C" {
+
+ts_status ts_moe_forward(ts_moe* h, const void* x, int batch, float* y, cudaStream_t stream) {
+    if (!h || batch < 0 || batch > h->max_batch) return TS_ERR_INVALID_ARG;
+    if (batch == 0) return TS_OK;
+    if (!x || !y) return TS_ERR_INVALID_ARG;
+    ts_status st = moe_layer(h, x, nullptr, batch, y, stream);
+    if (st == TS_OK) h->last_batch = batch;
+    return st;
+}
+
+ts_status ts_moe_stack_forward(ts_moe* const* layers, int n_layers, float* hres, int batch,
+                               cudaStream_t stream) {
+    if (!layers || n_layers < 0 || !hres || batch < 0) return TS_ERR_INVALID_ARG;
+    if (batch == 0 || n_layers == 0) return TS_OK;
+    for (int l = 0; l < n_layers; ++l) {
+        const ts_moe* h = layers[l];
+        if (!h || h->d != layers[0]->d || h->dt != layers[0]->dt || batch > h->max_batch)
+            return TS_ERR_INVALID_ARG;
+    }
+    for (int l = 0; l < n_layers; ++l) {
+        ts_status st = moe_layer(layers[l], nullptr, hres, batch, nullptr, stream);
+        if (st != TS_OK) return st;
+        layers[l]->last_batch = batch;
+    }
+    return TS_OK;
+}
+
+ts_status ts_moe_get_routing(ts_moe* h, cudaStream_t stream, int32_t* sel, float* w) {
+    if (!h || h->last_batch == 0) return TS_ERR_INVALID_ARG;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return TS_ERR_CUDA;
+    std::vector<TokenRoute> r(h->last_batch);
+    if (cudaMemcpy(r.data(), h->route, r.size() * sizeof(TokenRoute), cudaMemcpyDeviceToHost) !=
+        cudaSuccess)
+        return TS_ERR_CUDA;
+    for (int t = 0; t < h->last_batch; ++t)
+        for (int k = 0; k < h->top_k; ++k) {
+            if (sel) sel[t * h->top_k + k] = r[t].sel[k];
+            if (w) w[t * h->top_k + k] = r[t].w[k];
+        }
+    return TS_OK;
+}
+
+ts_status ts_moe_get_active(ts_moe* h, cudaStream_t stream, int expert, int token, int32_t* gate_idx,
+                            int* n_gate, int32_t* both_idx, int* n_both) {
+    if (!h || h->last_batch == 0 || expert < 0 || expert >= h->E) return TS_ERR_INVALID_ARG;
+    if (token < -1 || token >= h->last_batch) return TS_ERR_INVALID_ARG;
+    std::vector<int32_t> sel((size_t)h->last_batch * h->top_k);
+    ts_status st = ts_moe_get_routing(h, stream, sel.data(), nullptr);
+    if (st != TS_OK) return st;
+    // local token index of each routed token, in token order
+    std::vector<int> toks;
+    for (int t = 0; t < h->last_batch; ++t)
+        for (int k = 0; k < h->top_k; ++k)
+            if (sel[(size_t)t * h->top_k + k] == expert) toks.push_back(t);
+    const uint8_t* gb = h->s.gbits + (size_t)expert * kMaxPass * h->nbytes;
+    const uint8_t* bb = h->s.bbits + (size_t)expert * kMaxPass * h->nbytes;
+    if (token < 0)
+        return fetch_active(stream, gb, bb, h->nbytes, h->m, nullptr, 0, (int)toks.size(), gate_idx,
+                            n_gate, both_idx, n_both);
+    const auto it = std::find(toks.begin(), toks.end(), token);
+    if (it == toks.end()) {  // token not routed to this expert: nothing active
+        if (n_gate) *n_gate = 0;
+        if (n_both) *n_both = 0;
+        return TS_OK;
+    }
+    return fetch_active(stream, gb, bb, h->nbytes, h->m, nullptr, (int)(it - toks.begin()), 1,
+                        gate_idx, n_gate, both_idx, n_both);
+}
+
+ts_status ts_moe_get_error(ts_moe* h, cudaStream_t stream) {
+    if (!h) return TS_ERR_INVALID_ARG;
+    return read_status(h->s.status, stream);
+}
+
+// ---------------------------------------------------------------------------
+// graphs
+// ---------------------------------------------------------------------------
+}  // extern "C"
+
+namespace {
+
+template <typename F>
+ts_status capture(ts_graph** out, F&& body) {
+    if (!out) return TS_ERR_INVALID_ARG;
+    *out = nullptr;
+    cudaStream_t s;
+    if (cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking) != cudaSuccess) return TS_ERR_CUDA;
+    if (cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+        cudaStreamDestroy(s);
+        return TS_ERR_CUDA;
+    }
+    ts_status st = body(s);
+    cudaGraph_t g = nullptr;
+    const cudaError_t ec = cudaStreamEndCapture(s, &g);
+    cudaStreamDestroy(s);
+    if (st != TS_OK || ec != cudaSuccess) {
+        if (g) cudaGraphDestroy(g);
+        return st != TS_OK ? st : TS_ERR_CUDA;
+    }
+    ts_graph* gr = new (std::nothrow) ts_graph();
+    if (!gr) {
+        cudaGraphDestroy(g);
+        return TS_ERR_OOM;
+    }
+    gr->graph = g;
+    if (cudaGraphInstantiate(&gr->exec, g, 0) != cudaSuccess) {
+        cudaGraphDestroy(g);
+        delete gr;
+        return TS_ERR_CUDA;
+    }
+    *out = gr;
+    return TS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+ts_status ts_graph_capture_stack(ts_graph** out, ts_ffn* const* layers, int n_layers, float* h,
+                                 int batch, const int32_t* const* active_idx, const int* n_active) {
+    return capture(out, [&](cudaStream_t s) {
+        return ts_stack_forward(layers, n_layers, h, batch, s, active_idx, n_active);
+    });
+}
+
+ts_status ts_graph_capture_moe_stack(ts_graph** out, ts_moe* const* layers, int n_layers, float* h,
+                                     int batch) {
+    return capture(out, [&](cudaStream_t s) { return ts_moe_stack_forward(layers, n_layers, h, batch, s); });
+}
+
+ts_status ts_graph_launch(ts_graph* g, cudaStream_t stream) {
+    if (!g || !g->exec) return TS_ERR_INVALID_ARG;
+    return cuda_status(cudaGraphLaunch(g->exec, stream));
+}
+
+void ts_graph_destroy(ts_graph* g) {
+    if (!g) return;
+    if (g->exec) cudaGraphExecDestroy(g->exec);
+    if (g->graph) cudaGraphDestroy(g->graph);
+    delete g;
+}
+
+}  // extern "C"

@@ -1,0 +1,241 @@
+// ts_kernels.cuh -- device helpers and launch parameter blocks shared by the
+// sm_103a kernels of libtsffn (gate+up, down, router) and the C-ABI layer.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace tsffn {
+
+constexpr int kWarp = 32;
+constexpr int kChunk = 8;       // rows per gate/up work item (one bitmap byte)
+constexpr int kMaxPass = 8;     // tokens per pass of the CUDA-core kernels
+constexpr int kMaxBatch = 64;   // largest dense batch
+constexpr int kMaxMoeBatch = 8; // largest MoE batch
+constexpr int kMaxExperts = 16;
+constexpr int kMaxTopK = 4;
+constexpr int kColSlice = 256;  // output columns per down-projection CTA
+constexpr int kDownWarps = 8;
+constexpr int kGateUpWarps = 8;
+constexpr int kRouterMaxD = 16384;  // router keeps one fp32 activation row in shared memory
+
+// device status bits (OR-ed into the handle's status word)
+constexpr unsigned kStatusBadIndex = 1u;
+
+// Routing of one token: experts in selection order and their weights.
+struct TokenRoute {
+    int sel[kMaxTopK];
+    float w[kMaxTopK];
+};
+
+// Per-expert (or the single FFN's) weight rows, [m][d] neuron-major.
+struct ExpertPtrs {
+    const void* wg;
+    const void* wu;
+    const void* wd;
+};
+
+// Parameters of one gate+up launch (K1+K2 fused) and the matching down
+// launch (K3). `route == nullptr` means a single FFN whose experts[0] gets the
+// pass's tokens tok0 .. tok0+nt-1 with weight 1.
+struct FfnLaunch {
+    int d, m;
+    int n_rows;             // size of the row space: m, or the list length
+    const int32_t* rows;    // predictor list (ascending neuron ids) or nullptr
+    int batch;              // tokens of the whole call
+    int tok0, nt;           // this pass: tokens tok0 .. tok0+nt-1 (dense only)
+    const void* x;          // [batch][d] activations, weight dtype
+    float* h;               // [batch][d] residual (stack mode) or nullptr
+    float* y;               // [batch][d] output (forward mode)
+    int norm_from_h;        // 1: x = rmsnorm(h) computed in the gate+up prologue
+    int n_experts;
+    ExpertPtrs ex[kMaxExperts];
+    const TokenRoute* route;  // MoE routing [batch] or nullptr
+    int top_k;
+    // scratch
+    float* cval;            // [expert][kMaxPass][n_rows_cap]: routed w * c
+    int cval_tok_stride;    // n_rows_cap
+    uint8_t* gbits;         // per-token gate-active bitmap bytes
+    uint8_t* bbits;         // per-token both-active bitmap bytes
+    long long bits_expert_stride;  // bytes between experts (0 for a single FFN)
+    int bits_tok_base;      // token index of local token 0 in the bitmaps (tok0 for dense)
+    int nbytes;             // bitmap bytes per token (multiple of 4)
+    uint8_t* ubits;         // [expert][nbytes] union over the pass's tokens: both-active
+    uint8_t* ugbits;        // [expert][nbytes] union gate-active
+    float* partial;         // [n_rg][kMaxPass][d]
+    unsigned* counters;     // [n_cs]
+    unsigned* status;
+    int n_rg, n_cs;
+    int residual_out;       // 1: h += y instead of y =
+};
+
+struct RouterLaunch {
+    int d, n_experts, top_k, batch;
+    const void* x;          // [batch][d] or nullptr in norm mode
+    const float* h;         // [batch][d] residual (norm mode)
+    void* xbuf;             // [batch][d] normalised activations written in norm mode
+    const void* wr;         // [n_experts][d]
+    TokenRoute* route;      // [batch] out
+};
+
+// ---------------------------------------------------------------------------
+// device helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint4 ld_stream(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
+// Programmatic dependent launch: wait for the previous grid's results / let
+// the next grid start its independent prologue.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Asynchronous L2 prefetch of `bytes` (multiple of 16) at a 16-byte aligned address.
+__device__ __forceinline__ void prefetch_l2_bulk(const void* p, unsigned bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Elements of a 16-byte vector, as fp32.
+template <typename T>
+struct Vec;
+
+template <>
+struct Vec<float> {
+    static constexpr int N = 4;
+    __device__ __forceinline__ static void unpack(const uint4& v, float* o) {
+        o[0] = __uint_as_float(v.x);
+        o[1] = __uint_as_float(v.y);
+        o[2] = __uint_as_float(v.z);
+        o[3] = __uint_as_float(v.w);
+    }
+    __device__ __forceinline__ static float load1(const void* p, size_t i) {
+        return static_cast<const float*>(p)[i];
+    }
+    __device__ __forceinline__ static float round_act(float v) { return v; }
+    __device__ __forceinline__ static void store1(void* p, size_t i, float v) {
+        static_cast<float*>(p)[i] = v;
+    }
+};
+
+template <>
+struct Vec<__nv_bfloat16> {
+    static constexpr int N = 8;
+    __device__ __forceinline__ static void unpack(const uint4& v, float* o) {
+        o[0] = bf16lo(v.x); o[1] = bf16hi(v.x);
+        o[2] = bf16lo(v.y); o[3] = bf16hi(v.y);
+        o[4] = bf16lo(v.z); o[5] = bf16hi(v.z);
+        o[6] = bf16lo(v.w); o[7] = bf16hi(v.w);
+    }
+    __device__ __forceinline__ static float load1(const void* p, size_t i) {
+        return __bfloat162float(static_cast<const __nv_bfloat16*>(p)[i]);
+    }
+    __device__ __forceinline__ static float round_act(float v) {
+        return __bfloat162float(__float2bfloat16_rn(v));
+    }
+    __device__ __forceinline__ static void store1(void* p, size_t i, float v) {
+        static_cast<__nv_bfloat16*>(p)[i] = __float2bfloat16_rn(v);
+    }
+};
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Expert/token bookkeeping resolved by every CTA from the routing table.
+struct ExpertSets {
+    int n_act;                          // experts with at least one token
+    int act[kMaxExperts];               // their ids, ascending
+    int ntok[kMaxExperts];              // tokens per expert
+    int tok[kMaxExperts][kMaxMoeBatch];  // global token ids, ascending
+    float w[kMaxExperts][kMaxMoeBatch];  // routing weights
+};
+
+// Fill `s` (shared memory) from the launch; call with the whole block, ends
+// with __syncthreads(). Single FFN: one expert with tokens tok0..tok0+nt-1.
+__device__ __forceinline__ void resolve_experts(const FfnLaunch& a, ExpertSets& s) {
+    if (threadIdx.x < kWarp) {
+        const int lane = threadIdx.x;
+        if (a.route == nullptr) {
+            if (lane == 0) {
+                s.n_act = 1;
+                s.act[0] = 0;
+                s.ntok[0] = a.nt;
+            }
+            if (lane < a.nt) {
+                s.tok[0][lane] = a.tok0 + lane;
+                s.w[0][lane] = 1.0f;
+            }
+        } else {
+            // lane e collects the tokens routed to expert e, in token order
+            int n = 0;
+            if (lane < a.n_experts) {
+                for (int t = 0; t < a.batch; ++t) {
+                    const TokenRoute r = a.route[t];
+                    for (int k = 0; k < a.top_k; ++k) {
+                        if (r.sel[k] == lane && n < kMaxMoeBatch) {
+                            s.tok[lane][n] = t;
+                            s.w[lane][n] = r.w[k];
+                            ++n;
+                        }
+                    }
+                }
+                s.ntok[lane] = n;
+            }
+            const unsigned has = __ballot_sync(0xffffffffu, lane < a.n_experts && n > 0);
+            if (lane < a.n_experts && n > 0) s.act[__popc(has & ((1u << lane) - 1u))] = lane;
+            if (lane == 0) s.n_act = __popc(has);
+        }
+    }
+    __syncthreads();
+}
+
+// x = round(h / sqrt(mean(h^2) + 1e-5)), x[d-1] = 1, into shared memory.
+// Every block computes the same bits (fixed per-thread order, fixed tree).
+template <typename T>
+__device__ __forceinline__ void block_rmsnorm(const float* __restrict__ h, int d, float* __restrict__ out,
+                              float* red) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    float ss = 0.0f;
+    for (int i = threadIdx.x; i < d; i += blockDim.x) {
+        const float v = h[i];
+        ss = fmaf(v, v, ss);
+    }
+    ss = warp_sum(ss);
+    if (lane == 0) red[warp] = ss;
+    __syncthreads();
+    float tot = 0.0f;
+    for (int w = 0; w < nw; ++w) tot += red[w];
+    const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)d), 1e-5f));
+    for (int i = threadIdx.x; i < d; i += blockDim.x)
+        out[i] = (i == d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(h[i], rms));
+    __syncthreads();
+}
+
+}  // namespace tsffn
+
+// Host-side launchers (defined in the kernel translation units).
+namespace tsffn {
+cudaError_t launch_gate_up(const FfnLaunch& a, int wdtype, int pass_tokens, int grid,
+                           cudaStream_t stream, bool pdl);
+cudaError_t launch_down(const FfnLaunch& a, int wdtype, int pass_tokens, cudaStream_t stream,
+                        bool pdl);
+cudaError_t launch_router(const RouterLaunch& a, int wdtype, cudaStream_t stream, bool pdl);
+// Set per-kernel attributes once per device, before any launch or capture.
+cudaError_t prepare_gate_up(int optin_smem);
+cudaError_t prepare_down();
+cudaError_t prepare_router();
+// Resident gate+up CTAs per SM with `x_tokens` activation rows in shared memory.
+int gate_up_blocks_per_sm(int wdtype, int pass_tokens, int x_tokens, int d);
+}  // namespace tsffn

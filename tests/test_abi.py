@@ -1,0 +1,94 @@
+"""The C-ABI library loads without a GPU, exports every symbol include/ts_ffn.h
+declares, and rejects bad arguments before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "ts_ffn.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2406_05955_gb300 import binding, build
+
+    build.build()
+    return binding.lib()
+
+
+def _declared():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(ts_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_header_symbols_exported(lib):
+    from paper_2406_05955_gb300 import binding
+
+    names = _declared()
+    assert len(names) >= 20
+    raw = ctypes.CDLL(binding.LIB_PATH)
+    for n in names:
+        assert hasattr(raw, n), f"{n} declared in ts_ffn.h but not exported"
+    assert set(names) == set(binding.SIGNATURES), "binding signatures and header disagree"
+
+
+def test_status_strings_and_version(lib):
+    from paper_2406_05955_gb300 import binding
+
+    names = [binding.status_str(s) for s in range(7)]
+    assert names == ["TS_OK", "TS_ERR_INVALID_ARG", "TS_ERR_CUDA", "TS_ERR_OOM", "TS_ERR_BAD_INDEX",
+                     "TS_ERR_TIMEOUT", "TS_ERR_UNSUPPORTED"]
+    assert binding.status_str(99) == "TS_ERR_UNKNOWN"
+    assert lib.ts_version() >= 100
+
+
+def test_argument_validation_without_device(lib):
+    from paper_2406_05955_gb300.binding import TS_BF16, TS_ERR_INVALID_ARG, TS_F32
+
+    h = ctypes.c_void_p()
+    good = 0x10000
+    assert lib.ts_ffn_create(None, 64, 32, TS_BF16, good, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_create(ctypes.byref(h), 0, 32, TS_BF16, good, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_create(ctypes.byref(h), 64, 0, TS_BF16, good, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_create(ctypes.byref(h), 64, 32, 7, good, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_create(ctypes.byref(h), 64, 32, TS_BF16, None, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_create(ctypes.byref(h), 64, 32, TS_BF16, good + 2, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_create(ctypes.byref(h), 12, 32, TS_BF16, good, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_create(ctypes.byref(h), 6, 32, TS_F32, good, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_create(ctypes.byref(h), 64, 32, TS_BF16, good, good, good, 0) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_create(ctypes.byref(h), 64, 32, TS_BF16, good, good, good, 65) == TS_ERR_INVALID_ARG
+    assert h.value is None
+    assert lib.ts_ffn_forward(None, good, 1, good, None, None, 0) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_gate_up(None, good, 1, None, None, 0) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_down(None, 1, good, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_stack_forward(None, 1, good, 1, None, None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_get_active(None, None, 0, None, None, None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_get_error(None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_moe_create(None, 64, 8, 2, TS_BF16, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_moe_create(ctypes.byref(h), 64, 8, 5, TS_BF16, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_moe_create(ctypes.byref(h), 64, 17, 2, TS_BF16, good, good, 1) == TS_ERR_INVALID_ARG
+    assert lib.ts_moe_create(ctypes.byref(h), 64, 8, 2, TS_BF16, good, good, 9) == TS_ERR_INVALID_ARG
+    assert lib.ts_moe_forward(None, good, 1, good, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_moe_stack_forward(None, 1, good, 1, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_moe_get_routing(None, None, None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_moe_get_active(None, None, 0, 0, None, None, None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_moe_get_error(None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_graph_launch(None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_graph_capture_stack(None, None, 0, None, 0, None, None) == TS_ERR_INVALID_ARG
+    lib.ts_ffn_destroy(None)
+    lib.ts_moe_destroy(None)
+    lib.ts_graph_destroy(None)
+
+
+def test_binding_refuses_cpu_tensors():
+    """The product path has no CPU fallback: CPU tensors are an error."""
+    import torch
+
+    import paper_2406_05955_gb300 as ts
+
+    w = torch.zeros(8, 64, dtype=torch.bfloat16)
+    with pytest.raises(TypeError):
+        ts.Ffn(w, w, w)
