@@ -83,6 +83,11 @@ class Dist:
             self.pg.destroy_process_group()
 
 
+def whole_job_value(batch: int, steps: int, world: int, t_max: float) -> float:
+    """Tokens of every replica over the slowest replica's time (replicas run the same work)."""
+    return batch * steps * world / t_max
+
+
 # ---------------------------------------------------------------------------
 # clock sampling during the timed region
 # ---------------------------------------------------------------------------
@@ -142,8 +147,11 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # workload set-up
 # ---------------------------------------------------------------------------
-def make_stack(ts, wl, dev, batch: int, predictor: bool):
-    cfg = wl.WORKLOADS["mistral7b-ffn-stack-bf16-predictor" if predictor else "mistral7b-ffn-stack-bf16-b1-act10"]
+def make_stack(ts, wl, dev, batch: int, predictor: bool, n_layers: int | None = None):
+    cfg = dict(wl.WORKLOADS["mistral7b-ffn-stack-bf16-predictor" if predictor
+                            else "mistral7b-ffn-stack-bf16-b1-act10"])
+    if n_layers:
+        cfg["layers"] = n_layers
     d, m, n_layers = cfg["d"], cfg["m"], cfg["layers"]
     layers, ffns, lists = [], [], []
     for l in range(n_layers):
@@ -211,7 +219,7 @@ def dense_cublas_tokens_per_s(layers, batch, dev, steps=10) -> float:
             g = x @ L.w_gate.t()
             u = x @ L.w_up.t()
             c = torch.relu(g) * torch.relu(u)
-            hh = hh + (c @ L.w_down.t()).float()
+            hh = hh + (c @ L.w_down).float()  # W_down is neuron-major [m][d]
         return hh
 
     with torch.cuda.stream(stream):
@@ -270,7 +278,7 @@ def run_ours(args, dist: Dist) -> dict | None:
     torch.cuda.set_device(dev)
     B = args.batch
     predictor = args.workload == "predictor"
-    cfg, layers, ffns, lists = make_stack(ts, wl, dev, B, predictor)
+    cfg, layers, ffns, lists = make_stack(ts, wl, dev, B, predictor, args.layers)
     n_layers = cfg["layers"]
     h0 = wl.residual(B, cfg["d"], seed=cfg["seed"] - 1, device=dev)
     h = h0.clone()
@@ -291,7 +299,7 @@ def run_ours(args, dist: Dist) -> dict | None:
     dist.barrier()
     clk = clocks.stop()
     t_max = dist.max(elapsed)
-    value = B * args.steps * dist.world / t_max
+    value = whole_job_value(B, args.steps, dist.world, t_max)
 
     # end-to-end through the public API with host buffers (pinned), copies inside the timed region
     h_host = torch.empty_like(h0, device="cpu").pin_memory()
@@ -349,7 +357,7 @@ def run_ours(args, dist: Dist) -> dict | None:
                      "traffic": None, "bytes_per_launch": gate_up_bytes,
                      "avg_launch_us": t_gate_up * 1e6},
         "e2e": e2e,
-        "gpu_launches": 2 * n_layers * args.steps,
+        "gpu_launches": 2 * n_layers * args.steps * ((B + 7) // 8),
         "clocks": clk,
     }
     if not args.no_dense:
@@ -412,6 +420,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["stack", "predictor"], default="stack")
     ap.add_argument("--batch", type=int, default=1)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="fewer layers than the workload's 32 (profiling cases only; not a bench line)")
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()

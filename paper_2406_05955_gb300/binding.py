@@ -111,13 +111,27 @@ def _stream(stream) -> int:
     return int(stream)
 
 
+_EMPTY_LISTS: dict = {}
+
+
 def _list(active_idx):
+    """(device pointer, length) of a predictor list; None means detected mode.
+
+    An empty CUDA tensor has a null data pointer, which the C ABI reads as "no
+    list", so an empty list is passed as a valid one-element buffer of length 0.
+    """
     if active_idx is None:
         return None, 0
     _dev(active_idx, "active_idx")
     if active_idx.dtype != torch.int32:
         raise TypeError("active_idx must be int32")
-    return active_idx.data_ptr(), int(active_idx.numel())
+    n = int(active_idx.numel())
+    if n == 0:
+        dev = active_idx.device
+        if dev not in _EMPTY_LISTS:
+            _EMPTY_LISTS[dev] = torch.zeros(1, dtype=torch.int32, device=dev)
+        return _EMPTY_LISTS[dev].data_ptr(), 0
+    return active_idx.data_ptr(), n
 
 
 class Ffn:

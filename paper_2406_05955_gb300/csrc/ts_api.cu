@@ -69,21 +69,16 @@ ts_status alloc_arena(Arena* ar) {
     return TS_OK;
 }
 
-// Scratch of the grouped kernels: per-expert c values and bitmaps, the down
-// projection's partials and tickets, and the device status word.
+// Scratch of the grouped kernels: per-expert c values and bitmaps, and the
+// device status word.
 struct Scratch {
     float* cval = nullptr;
     uint8_t* gbits = nullptr;
     uint8_t* bbits = nullptr;
     uint8_t* ubits = nullptr;
     uint8_t* ugbits = nullptr;
-    float* partial = nullptr;
-    unsigned* counters = nullptr;
     unsigned* status = nullptr;
 };
-
-int down_col_slices(int d) { return (d + kColSlice - 1) / kColSlice; }
-int down_row_groups(int d, int num_sms) { return std::max(1, 2 * num_sms / down_col_slices(d)); }
 
 }  // namespace
 
@@ -94,7 +89,7 @@ struct ts_ffn {
     const void* wu = nullptr;
     const void* wd = nullptr;
     DeviceInfo dev;
-    int n_cs = 0, n_rg = 0, nbytes = 0;
+    int nbytes = 0;
     Arena arena;
     Scratch s;
     int grid[9] = {0};  // gate+up grid per pass width 1, 2, 4, 8
@@ -110,7 +105,7 @@ struct ts_moe {
     const void* wr = nullptr;
     ExpertPtrs ex[kMaxExperts];
     DeviceInfo dev;
-    int n_cs = 0, n_rg = 0, nbytes = 0;
+    int nbytes = 0;
     Arena arena;
     Scratch s;
     TokenRoute* route = nullptr;
@@ -168,16 +163,12 @@ ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void*
     h->wu = w_up;
     h->wd = w_down;
     h->dev = dev;
-    h->n_cs = down_col_slices(d);
-    h->n_rg = down_row_groups(d, dev.num_sms);
     h->nbytes = (m + 31) / 32 * 4;
     const size_t o_cval = h->arena.take((size_t)kMaxPass * m * sizeof(float));
     const size_t o_g = h->arena.take((size_t)max_batch * h->nbytes);
     const size_t o_b = h->arena.take((size_t)max_batch * h->nbytes);
     const size_t o_u = h->arena.take((size_t)h->nbytes);
     const size_t o_ug = h->arena.take((size_t)h->nbytes);
-    const size_t o_p = h->arena.take((size_t)h->n_rg * kMaxPass * d * sizeof(float));
-    const size_t o_c = h->arena.take((size_t)h->n_cs * sizeof(unsigned));
     const size_t o_s = h->arena.take(sizeof(unsigned));
     st = alloc_arena(&h->arena);
     if (st != TS_OK) {
@@ -189,8 +180,6 @@ ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void*
     h->s.bbits = h->arena.at<uint8_t>(o_b);
     h->s.ubits = h->arena.at<uint8_t>(o_u);
     h->s.ugbits = h->arena.at<uint8_t>(o_ug);
-    h->s.partial = h->arena.at<float>(o_p);
-    h->s.counters = h->arena.at<unsigned>(o_c);
     h->s.status = h->arena.at<unsigned>(o_s);
     const int n_chunks = (m + kChunk - 1) / kChunk;
     for (int nt : {1, 2, 4, 8}) {
@@ -232,11 +221,7 @@ FfnLaunch ffn_launch(const ts_ffn* h, int batch, const int32_t* rows, int n_rows
     a.nbytes = h->nbytes;
     a.ubits = h->s.ubits;
     a.ugbits = h->s.ugbits;
-    a.partial = h->s.partial;
-    a.counters = h->s.counters;
     a.status = h->s.status;
-    a.n_rg = h->n_rg;
-    a.n_cs = h->n_cs;
     return a;
 }
 
@@ -445,8 +430,6 @@ ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype 
     h->wr = w_router;
     for (int e = 0; e < n_experts; ++e) h->ex[e] = ExpertPtrs{experts[e]->wg, experts[e]->wu, experts[e]->wd};
     h->dev = dev;
-    h->n_cs = down_col_slices(d);
-    h->n_rg = down_row_groups(d, dev.num_sms);
     h->nbytes = (h->m + 31) / 32 * 4;
     const int m = h->m, E = n_experts;
     const size_t o_cval = h->arena.take((size_t)E * kMaxPass * m * sizeof(float));
@@ -454,8 +437,6 @@ ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype 
     const size_t o_b = h->arena.take((size_t)E * kMaxPass * h->nbytes);
     const size_t o_u = h->arena.take((size_t)E * h->nbytes);
     const size_t o_ug = h->arena.take((size_t)E * h->nbytes);
-    const size_t o_p = h->arena.take((size_t)h->n_rg * kMaxPass * d * sizeof(float));
-    const size_t o_c = h->arena.take((size_t)h->n_cs * sizeof(unsigned));
     const size_t o_s = h->arena.take(sizeof(unsigned));
     const size_t o_r = h->arena.take((size_t)max_batch * sizeof(TokenRoute));
     const size_t o_x = h->arena.take((size_t)max_batch * d * elem_size(wdtype));
@@ -469,8 +450,6 @@ ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype 
     h->s.bbits = h->arena.at<uint8_t>(o_b);
     h->s.ubits = h->arena.at<uint8_t>(o_u);
     h->s.ugbits = h->arena.at<uint8_t>(o_ug);
-    h->s.partial = h->arena.at<float>(o_p);
-    h->s.counters = h->arena.at<unsigned>(o_c);
     h->s.status = h->arena.at<unsigned>(o_s);
     h->route = h->arena.at<TokenRoute>(o_r);
     h->xbuf = h->arena.at<void>(o_x);
@@ -538,11 +517,7 @@ ts_status moe_layer(ts_moe* h, const void* x, float* hres, int batch, float* y, 
     a.nbytes = h->nbytes;
     a.ubits = h->s.ubits;
     a.ugbits = h->s.ugbits;
-    a.partial = h->s.partial;
-    a.counters = h->s.counters;
     a.status = h->s.status;
-    a.n_rg = h->n_rg;
-    a.n_cs = h->n_cs;
     const int w = pow2_tokens(batch);
     st = cuda_status(launch_gate_up(a, h->dt, w, h->grid[w], stream, true));
     if (st != TS_OK) return st;

@@ -2,22 +2,27 @@
 // (the "Combined(x) W_down" of Eq. 1, restricted to the non-zero dReLU
 // activations of Eq. 2).
 //
-// Grid (n_cs, n_rg): blockIdx.x picks a slice of kColSlice output columns,
-// blockIdx.y one of n_rg equal shares of the ordered active list. The list is
-// not materialised in global memory: every CTA reads the union bitmap words
-// (expert-major, row order), prefix-sums their popcounts and pulls out the
-// entries of its share. Each warp takes every kDownWarps-th entry and reads
-// that row's 512-byte (bf16) or 1 KB (fp32) column segment with 16-byte
-// loads, accumulating c * w in fp32 registers per token. The CTA sums its
-// warps in shared memory, writes one partial per (share, token, column), and
-// the last CTA of the column slice to finish (atomic ticket) adds the n_rg
-// partials in share order -- a fixed order, so y is bitwise reproducible.
+// One CTA per slice of kDownCols output columns: 64 bytes of every active
+// row (32 bf16 or 16 fp32 columns). Every CTA reads the union bitmap words
+// (expert-major, row order), prefix-sums their popcounts and stages the
+// ordered (expert, row) entries in shared memory. A warp instruction covers
+// 8 entries (4 lanes x 16 bytes per row segment); each warp keeps up to 16
+// such instructions in flight, accumulating c * w in fp32 registers per
+// batch slot. Rows are reduced across lanes (shuffles) and warps (shared
+// memory) in a fixed order and written straight to y (or added to the
+// residual): no partial buffers, no cross-CTA hand-off, bitwise reproducible.
 #include "ts_kernels.cuh"
 
 namespace tsffn {
 
-constexpr int kListCap = 1024;  // entries a CTA stages in shared memory at once
-constexpr int kDownUnroll = 4;  // rows a warp has in flight
+constexpr int kListCap = 2048;  // entries a CTA stages in shared memory at once
+constexpr int kLanesPerRow = 4;
+constexpr int kRowsPerInst = kWarp / kLanesPerRow;  // 8
+
+template <int NT>
+struct DownShape {
+    static constexpr int U = NT <= 2 ? 16 : (NT == 4 ? 8 : 4);  // row groups in flight per warp
+};
 
 __device__ __forceinline__ unsigned union_word(const FfnLaunch& a, const ExpertSets& es,
                                                int nwords, int w) {
@@ -33,14 +38,13 @@ __device__ __forceinline__ unsigned union_word(const FfnLaunch& a, const ExpertS
 template <typename T, int NT>
 __global__ void __launch_bounds__(kDownWarps * kWarp) k_down(const FfnLaunch a) {
     constexpr int VEC = Vec<T>::N;
-    constexpr int V = kColSlice / (kWarp * VEC);  // 16-byte loads per lane per row
-    constexpr int VPL = V * VEC;                  // columns per lane
-    extern __shared__ __align__(16) float red[];  // [kDownWarps][NT][kColSlice]
+    constexpr int COLS = kLanesPerRow * VEC;  // columns per CTA (64 bytes of a row)
+    constexpr int U = DownShape<NT>::U;
     __shared__ ExpertSets es;
     __shared__ int2 s_list[kListCap];
     __shared__ int s_scan[kDownWarps];
     __shared__ int s_total;
-    __shared__ int s_last;
+    __shared__ float red[kDownWarps][NT][COLS];
 
     pdl_wait();
     pdl_launch_dependents();
@@ -51,11 +55,9 @@ __global__ void __launch_bounds__(kDownWarps * kWarp) k_down(const FfnLaunch a) 
     const int tid = threadIdx.x;
     const int nthr = blockDim.x;
     const int d = a.d;
-    const int cs = blockIdx.x;
-    const int rg = blockIdx.y;
-    const int n_rg = gridDim.y;
     const int nwords = (a.n_rows + 31) / 32;
     const int total_words = es.n_act * nwords;
+    const int n_slots = a.route ? a.batch : a.nt;
 
     // contiguous word range per thread, popcount, block exclusive scan
     const int per = (total_words + nthr - 1) / nthr;
@@ -83,19 +85,17 @@ __global__ void __launch_bounds__(kDownWarps * kWarp) k_down(const FfnLaunch a) 
     __syncthreads();
     const int off = s_scan[warp] + incl - cnt;  // rank of this thread's first entry
     const int N = s_total;
-    const int r0 = (int)((long long)N * rg / n_rg);
-    const int r1 = (int)((long long)N * (rg + 1) / n_rg);
 
-    // local token slot of each (expert, token): route ? global token : pass-local index
-    float acc[NT][VPL];
+    const int col = blockIdx.x * COLS + (lane & (kLanesPerRow - 1)) * VEC;
+    const int slot_in_inst = lane / kLanesPerRow;
+    float acc[NT][VEC];
 #pragma unroll
     for (int k = 0; k < NT; ++k)
 #pragma unroll
-        for (int c = 0; c < VPL; ++c) acc[k][c] = 0.0f;
+        for (int c = 0; c < VEC; ++c) acc[k][c] = 0.0f;
 
-    const int col_base = cs * kColSlice;
-    for (int s = r0; s < r1; s += kListCap) {
-        const int s1 = min(s + kListCap, r1);
+    for (int s = 0; s < N; s += kListCap) {
+        const int s1 = min(s + kListCap, N);
         if (cnt > 0 && off < s1 && off + cnt > s) {
             int rank = off;
             for (int w = w0; w < w1 && rank < s1; ++w) {
@@ -105,8 +105,7 @@ __global__ void __launch_bounds__(kDownWarps * kWarp) k_down(const FfnLaunch a) 
                     bits &= bits - 1u;
                     if (rank >= s) {
                         const int ea = w / nwords;
-                        const int pos = (w - ea * nwords) * 32 + b;
-                        s_list[rank - s] = make_int2(ea, pos);
+                        s_list[rank - s] = make_int2(ea, (w - ea * nwords) * 32 + b);
                     }
                     ++rank;
                 }
@@ -114,114 +113,82 @@ __global__ void __launch_bounds__(kDownWarps * kWarp) k_down(const FfnLaunch a) 
         }
         __syncthreads();
         const int n = s1 - s;
-        for (int i0 = warp; i0 < n; i0 += kDownWarps * kDownUnroll) {
-            uint4 wv[kDownUnroll][V];
-            int ent_e[kDownUnroll], ent_p[kDownUnroll];
+        const int n_inst = (n + kRowsPerInst - 1) / kRowsPerInst;
+        for (int g0 = warp; g0 < n_inst; g0 += kDownWarps * U) {
+            uint4 wv[U];
+            float cv[U][NT];
 #pragma unroll
-            for (int q = 0; q < kDownUnroll; ++q) {
-                const int i = i0 + q * kDownWarps;
-                ent_e[q] = -1;
-                ent_p[q] = 0;
+            for (int u = 0; u < U; ++u) {
+                const int i = (g0 + u * kDownWarps) * kRowsPerInst + slot_in_inst;
+                wv[u] = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+                for (int k = 0; k < NT; ++k) cv[u][k] = 0.0f;
                 if (i < n) {
                     const int2 en = s_list[i];
                     const int e = es.act[en.x];
-                    ent_e[q] = e;
-                    ent_p[q] = en.y;
                     const int j = a.rows ? a.rows[en.y] : en.y;
-                    const T* row = static_cast<const T*>(a.ex[e].wd) + (size_t)j * d;
+                    if (col < d)
+                        wv[u] = ld_stream(static_cast<const T*>(a.ex[e].wd) + (size_t)j * d + col);
+                    const float* cp = a.cval + ((size_t)e * kMaxPass) * a.cval_tok_stride + en.y;
 #pragma unroll
-                    for (int v = 0; v < V; ++v) {
-                        const int col = col_base + v * kWarp * VEC + lane * VEC;
-                        wv[q][v] = col < d ? ld_stream(row + col) : make_uint4(0u, 0u, 0u, 0u);
-                    }
-                } else {
-#pragma unroll
-                    for (int v = 0; v < V; ++v) wv[q][v] = make_uint4(0u, 0u, 0u, 0u);
+                    for (int k = 0; k < NT; ++k)
+                        if (k < n_slots) cv[u][k] = cp[(size_t)k * a.cval_tok_stride];
                 }
             }
 #pragma unroll
-            for (int q = 0; q < kDownUnroll; ++q) {
-                const int e = ent_e[q];
-                if (e < 0) continue;
-                const int ntok = es.ntok[e];
-                const float* cv = a.cval + ((size_t)e * kMaxPass) * a.cval_tok_stride + ent_p[q];
-                float f[V][VEC];
+            for (int u = 0; u < U; ++u) {
+                float f[VEC];
+                Vec<T>::unpack(wv[u], f);
 #pragma unroll
-                for (int v = 0; v < V; ++v) Vec<T>::unpack(wv[q][v], f[v]);
+                for (int k = 0; k < NT; ++k)
 #pragma unroll
-                for (int k = 0; k < NT; ++k) {
-                    if (k < ntok) {
-                        const float c = cv[(size_t)k * a.cval_tok_stride];
-                        const int slot = a.route ? es.tok[e][k] : k;
-                        // slot < NT always: MoE batches are <= NT tokens, passes are NT wide
-#pragma unroll
-                        for (int s2 = 0; s2 < NT; ++s2) {
-                            if (s2 == slot) {
-#pragma unroll
-                                for (int v = 0; v < V; ++v)
-#pragma unroll
-                                    for (int c2 = 0; c2 < VEC; ++c2)
-                                        acc[s2][v * VEC + c2] = fmaf(c, f[v][c2], acc[s2][v * VEC + c2]);
-                            }
-                        }
-                    }
-                }
+                    for (int c = 0; c < VEC; ++c) acc[k][c] = fmaf(cv[u][k], f[c], acc[k][c]);
             }
         }
         __syncthreads();
     }
 
-    // block reduction over warps (fixed order) -> partial of this share
-    const int n_slots = a.route ? a.batch : a.nt;
+    // reduce over the 8 row slots of a warp (lanes with equal lane % 4), then over warps
 #pragma unroll
     for (int k = 0; k < NT; ++k)
 #pragma unroll
-        for (int v = 0; v < V; ++v)
+        for (int c = 0; c < VEC; ++c) {
+            float v = acc[k][c];
+            v += __shfl_xor_sync(0xffffffffu, v, 4);
+            v += __shfl_xor_sync(0xffffffffu, v, 8);
+            v += __shfl_xor_sync(0xffffffffu, v, 16);
+            acc[k][c] = v;
+        }
+    if (lane < kLanesPerRow) {
 #pragma unroll
-            for (int c2 = 0; c2 < VEC; ++c2)
-                red[((size_t)warp * NT + k) * kColSlice + v * kWarp * VEC + lane * VEC + c2] =
-                    acc[k][v * VEC + c2];
-    __syncthreads();
-    for (int idx = tid; idx < n_slots * kColSlice; idx += nthr) {
-        const int k = idx / kColSlice;
-        const int c = idx - k * kColSlice;
-        const int col = col_base + c;
-        if (col >= d) continue;
-        float sum = 0.0f;
-        for (int w = 0; w < kDownWarps; ++w) sum += red[((size_t)w * NT + k) * kColSlice + c];
-        a.partial[((size_t)rg * kMaxPass + k) * d + col] = sum;
-    }
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) {
-        const unsigned prev = atomicAdd(&a.counters[cs], 1u);
-        s_last = (prev == (unsigned)(n_rg - 1));
+        for (int k = 0; k < NT; ++k)
+#pragma unroll
+            for (int c = 0; c < VEC; ++c) red[warp][k][lane * VEC + c] = acc[k][c];
     }
     __syncthreads();
-    if (!s_last) return;
-    __threadfence();
-    for (int idx = tid; idx < n_slots * kColSlice; idx += nthr) {
-        const int k = idx / kColSlice;
-        const int c = idx - k * kColSlice;
-        const int col = col_base + c;
-        if (col >= d) continue;
+    for (int idx = tid; idx < n_slots * COLS; idx += nthr) {
+        const int k = idx / COLS;
+        const int c = idx - k * COLS;
+        const int cc = blockIdx.x * COLS + c;
+        if (cc >= d) continue;
         float sum = 0.0f;
-        for (int r = 0; r < n_rg; ++r) sum += __ldcg(&a.partial[((size_t)r * kMaxPass + k) * d + col]);
+#pragma unroll
+        for (int w = 0; w < kDownWarps; ++w) sum += red[w][k][c];
         const int tok = a.route ? k : a.tok0 + k;
         if (a.residual_out)
-            a.h[(size_t)tok * d + col] += sum;
+            a.h[(size_t)tok * d + cc] += sum;
         else
-            a.y[(size_t)tok * d + col] = sum;
+            a.y[(size_t)tok * d + cc] = sum;
     }
-    if (tid == 0) a.counters[cs] = 0u;  // ticket ready for the next launch
 }
 
 template <typename T, int NT>
 static cudaError_t launch_t(const FfnLaunch& a, cudaStream_t stream, bool pdl) {
+    constexpr int COLS = kLanesPerRow * Vec<T>::N;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(a.n_cs, a.n_rg);
+    cfg.gridDim = dim3((a.d + COLS - 1) / COLS);
     cfg.blockDim = dim3(kDownWarps * kWarp);
-    cfg.dynamicSmemBytes = (size_t)kDownWarps * NT * kColSlice * sizeof(float);
+    cfg.dynamicSmemBytes = 0;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -231,24 +198,7 @@ static cudaError_t launch_t(const FfnLaunch& a, cudaStream_t stream, bool pdl) {
     return cudaLaunchKernelEx(&cfg, k_down<T, NT>, a);
 }
 
-template <typename T, int NT>
-static cudaError_t prepare_t() {
-    return cudaFuncSetAttribute(k_down<T, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)(kDownWarps * NT * kColSlice * sizeof(float)));
-}
-
-cudaError_t prepare_down() {
-    cudaError_t e = cudaSuccess;
-    if (e == cudaSuccess) e = prepare_t<__nv_bfloat16, 1>();
-    if (e == cudaSuccess) e = prepare_t<__nv_bfloat16, 2>();
-    if (e == cudaSuccess) e = prepare_t<__nv_bfloat16, 4>();
-    if (e == cudaSuccess) e = prepare_t<__nv_bfloat16, 8>();
-    if (e == cudaSuccess) e = prepare_t<float, 1>();
-    if (e == cudaSuccess) e = prepare_t<float, 2>();
-    if (e == cudaSuccess) e = prepare_t<float, 4>();
-    if (e == cudaSuccess) e = prepare_t<float, 8>();
-    return e;
-}
+cudaError_t prepare_down() { return cudaSuccess; }
 
 cudaError_t launch_down(const FfnLaunch& a, int wdtype, int pass_tokens, cudaStream_t stream,
                         bool pdl) {

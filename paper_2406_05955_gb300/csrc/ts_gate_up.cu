@@ -21,7 +21,7 @@ namespace tsffn {
 // accumulators stay in registers.
 template <typename T, int NT>
 struct GateUpShape {
-    static constexpr int R = NT == 1 ? 8 : (NT == 2 ? 4 : (NT == 4 ? 2 : 1));
+    static constexpr int R = NT == 1 ? 1 : (NT == 2 ? 4 : (NT == 4 ? 2 : 1));
     static constexpr int U = (sizeof(T) == 2 ? 16 : 8) / R;  // R <= 8, so U >= 1
 };
 
@@ -235,13 +235,26 @@ k_gate_up(const FfnLaunch a, int prefetch_rows) {
             a.ubits[(size_t)e * a.nbytes + chunk] = (uint8_t)ub;
             a.ugbits[(size_t)e * a.nbytes + chunk] = (uint8_t)gm;
         }
+        // c by batch slot: the pass-local token (single FFN) or the global
+        // token (MoE, 0 for tokens not routed to this expert)
         if (lane < kChunk && ((ub >> lane) & 1u)) {
             float* cv = a.cval + ((size_t)e * kMaxPass) * a.cval_tok_stride + p0 + lane;
+            float val[NT];
 #pragma unroll
-            for (int k = 0; k < NT; ++k) {
-                if (k < ntok) {
-                    const bool bk = greg[k] > 0.0f && ureg[k] > 0.0f;
-                    cv[(size_t)k * a.cval_tok_stride] = bk ? es.w[e][k] * (greg[k] * ureg[k]) : 0.0f;
+            for (int k = 0; k < NT; ++k)
+                val[k] = (k < ntok && greg[k] > 0.0f && ureg[k] > 0.0f) ? es.w[e][k] * (greg[k] * ureg[k])
+                                                                         : 0.0f;
+            if (a.route == nullptr) {
+#pragma unroll
+                for (int k = 0; k < NT; ++k)
+                    if (k < ntok) cv[(size_t)k * a.cval_tok_stride] = val[k];
+            } else {
+                for (int t = 0; t < a.batch; ++t) {
+                    float v = 0.0f;
+#pragma unroll
+                    for (int k = 0; k < NT; ++k)
+                        if (k < ntok && es.tok[e][k] == t) v = val[k];
+                    cv[(size_t)t * a.cval_tok_stride] = v;
                 }
             }
         }

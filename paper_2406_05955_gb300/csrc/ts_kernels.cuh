@@ -15,13 +15,16 @@ constexpr int kMaxBatch = 64;   // largest dense batch
 constexpr int kMaxMoeBatch = 8; // largest MoE batch
 constexpr int kMaxExperts = 16;
 constexpr int kMaxTopK = 4;
-constexpr int kColSlice = 256;  // output columns per down-projection CTA
 constexpr int kDownWarps = 8;
 constexpr int kGateUpWarps = 8;
 constexpr int kRouterMaxD = 16384;  // router keeps one fp32 activation row in shared memory
 
 // device status bits (OR-ed into the handle's status word)
 constexpr unsigned kStatusBadIndex = 1u;
+constexpr unsigned kStatusTimeout = 2u;
+// Bound on any device-side wait: a wait that lasts longer records
+// kStatusTimeout and the kernel winds down instead of hanging.
+constexpr unsigned long long kWaitLimitNs = 1000000000ull;
 
 // Routing of one token: experts in selection order and their weights.
 struct TokenRoute {
@@ -37,7 +40,8 @@ struct ExpertPtrs {
 };
 
 // Parameters of one gate+up launch (K1+K2 fused) and the matching down
-// launch (K3). `route == nullptr` means a single FFN whose experts[0] gets the
+// launch (K3). A batch slot is the pass-local token (single FFN) or the
+// global token (MoE). `route == nullptr` means a single FFN whose experts[0] gets the
 // pass's tokens tok0 .. tok0+nt-1 with weight 1.
 struct FfnLaunch {
     int d, m;
@@ -54,7 +58,7 @@ struct FfnLaunch {
     const TokenRoute* route;  // MoE routing [batch] or nullptr
     int top_k;
     // scratch
-    float* cval;            // [expert][kMaxPass][n_rows_cap]: routed w * c
+    float* cval;            // [expert][batch slot][n_rows_cap]: routed w * c at union rows
     int cval_tok_stride;    // n_rows_cap
     uint8_t* gbits;         // per-token gate-active bitmap bytes
     uint8_t* bbits;         // per-token both-active bitmap bytes
@@ -63,10 +67,7 @@ struct FfnLaunch {
     int nbytes;             // bitmap bytes per token (multiple of 4)
     uint8_t* ubits;         // [expert][nbytes] union over the pass's tokens: both-active
     uint8_t* ugbits;        // [expert][nbytes] union gate-active
-    float* partial;         // [n_rg][kMaxPass][d]
-    unsigned* counters;     // [n_cs]
     unsigned* status;
-    int n_rg, n_cs;
     int residual_out;       // 1: h += y instead of y =
 };
 
@@ -100,6 +101,67 @@ __device__ __forceinline__ void pdl_launch_dependents() {
 // Asynchronous L2 prefetch of `bytes` (multiple of 16) at a 16-byte aligned address.
 __device__ __forceinline__ void prefetch_l2_bulk(const void* p, unsigned bytes) {
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+// ---- shared-memory barriers and 1-D bulk copies (TMA) ----------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, unsigned count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, unsigned bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, unsigned parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Wait for the phase with the given parity to complete, for at most
+// kWaitLimitNs; false on timeout (the caller records it and winds down).
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait(bar, parity))
+        if (global_ns() - t0 > kWaitLimitNs) return false;
+    return true;
+}
+// 1-D bulk copy global -> this CTA's shared memory, completing on `bar`.
+__device__ __forceinline__ void tma_load_1d(void* dst, const void* src, unsigned bytes, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+__device__ __forceinline__ uint4 lds128(const void* p) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(smem_u32(p)));
+    return v;
+}
+__device__ __forceinline__ void named_bar_sync(int id, int threads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
 __device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }

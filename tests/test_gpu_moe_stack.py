@@ -179,7 +179,14 @@ def test_moe_stack_teacher_forced(ts, B):
 
 
 def test_mistral_stack_32_layers_graph(ts):
-    """The benchmark's workload and launch configuration: 32 layers in one graph, batch 1."""
+    """The benchmark's workload and launch configuration: 32 layers in one graph, batch 1.
+
+    The graph must give the same bits as direct launches; sampled layers are
+    compared with the oracle teacher-forced (the GPU gets the oracle's residual
+    at that layer). The free-running divergence over 32 layers -- bf16
+    re-rounding of the normalised activations amplified through the stack,
+    which neither side can avoid -- is bounded loosely as a gross-error check.
+    """
     cfg = wl.WORKLOADS["mistral7b-ffn-stack-bf16-b1-act10"]
     d, m, n_layers = cfg["d"], cfg["m"], cfg["layers"]
     dev = torch.device("cuda")
@@ -190,13 +197,25 @@ def test_mistral_stack_32_layers_graph(ts):
     hg = h0.clone()
     g = ts.Graph.stack(ffns, hg)
     g.launch()
+    hd = h0.clone()
+    ts.stack_forward(ffns, hd)
     torch.cuda.synchronize()
-    # free-running oracle stack over the same weights
-    st = oracle.stack(h0.cpu().numpy(), [(L.w_gate.cpu(), L.w_up.cpu(), L.w_down.cpu()) for L in layers],
-                      record=False)
+    assert torch.equal(hg, hd), "graph replay and direct launches differ"
+    assert all(f.get_error() == 0 for f in ffns)
+
+    host = [(L.w_gate.cpu(), L.w_up.cpu(), L.w_down.cpu()) for L in layers]
+    st = oracle.stack(h0.cpu().numpy(), host, record=True)
+    for l in (0, 1, 15, 31):
+        rec = st["layers"][l]
+        ref = oracle.ffn(rec["x"], *host[l])
+        hl = torch.from_numpy(rec["h_in"].copy()).to(dev)
+        ts.stack_forward([ffns[l]], hl)
+        y_gpu = hl.double().cpu().numpy() - rec["h_in"].astype(np.float64)
+        check_y(y_gpu, ref["y"], "bf16", f"layer {l}")
+        check_sets(*ffns[l].get_active(0), ref, 0)
+
     dy_gpu = hg.double().cpu().numpy() - h0.double().cpu().numpy()
     dy_ref = st["h"].astype(np.float64) - h0.double().cpu().numpy()
     err = rel_l2(dy_gpu, dy_ref)
-    assert err <= 2e-3, f"32-layer accumulated FFN output: rel L2 {err:.3e}"
-    # the last layer's active set against the oracle's, on the GPU's own input to it
-    assert ffns[-1].get_error() == 0
+    print(f"free-running 32-layer divergence of h_32 - h_0: rel L2 {err:.3e}")
+    assert err <= 2e-2, f"32-layer accumulated FFN output: rel L2 {err:.3e}"
