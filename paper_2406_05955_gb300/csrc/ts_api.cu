@@ -151,7 +151,12 @@ ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void*
     ts_status st = device_info(&dev);
     if (st != TS_OK) return st;
     const int pass_cap = std::min(max_batch, kMaxPass);
-    if ((size_t)pass_cap * d * sizeof(float) + 4096 > (size_t)dev.optin_smem) return TS_ERR_UNSUPPORTED;
+    {
+        int slots, slot_bytes, xs_stride;
+        size_t smem;
+        if (gate_up_config(wdtype, d, pass_cap, dev.optin_smem, &slots, &slot_bytes, &xs_stride, &smem) != 0)
+            return TS_ERR_UNSUPPORTED;
+    }
 
     ts_ffn* h = new (std::nothrow) ts_ffn();
     if (!h) return TS_ERR_OOM;
@@ -182,11 +187,7 @@ ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void*
     h->s.ugbits = h->arena.at<uint8_t>(o_ug);
     h->s.status = h->arena.at<unsigned>(o_s);
     const int n_chunks = (m + kChunk - 1) / kChunk;
-    for (int nt : {1, 2, 4, 8}) {
-        const int per_sm = gate_up_blocks_per_sm(wdtype, nt, nt, d);
-        const int need = (n_chunks + kGateUpWarps - 1) / kGateUpWarps;
-        h->grid[nt] = std::max(1, std::min(per_sm * dev.num_sms, need));
-    }
+    for (int nt : {1, 2, 4, 8}) h->grid[nt] = std::max(1, std::min(dev.num_sms, n_chunks));
     *out = h;
     return TS_OK;
 }
@@ -417,7 +418,12 @@ ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype 
     DeviceInfo dev;
     ts_status st = device_info(&dev);
     if (st != TS_OK) return st;
-    if ((size_t)max_batch * d * sizeof(float) + 4096 > (size_t)dev.optin_smem) return TS_ERR_UNSUPPORTED;
+    {
+        int slots, slot_bytes, xs_stride;
+        size_t smem;
+        if (gate_up_config(wdtype, d, max_batch, dev.optin_smem, &slots, &slot_bytes, &xs_stride, &smem) != 0)
+            return TS_ERR_UNSUPPORTED;
+    }
 
     ts_moe* h = new (std::nothrow) ts_moe();
     if (!h) return TS_ERR_OOM;
@@ -454,12 +460,8 @@ ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype 
     h->route = h->arena.at<TokenRoute>(o_r);
     h->xbuf = h->arena.at<void>(o_x);
     const int n_chunks = (m + kChunk - 1) / kChunk;
-    for (int nt : {1, 2, 4, 8}) {
-        const int x_tokens = std::min(nt, max_batch);
-        const int per_sm = gate_up_blocks_per_sm(wdtype, nt, x_tokens, d);
-        const int need = (std::min(E, nt * top_k) * n_chunks + kGateUpWarps - 1) / kGateUpWarps;
-        h->grid[nt] = std::max(1, std::min(per_sm * dev.num_sms, need));
-    }
+    for (int nt : {1, 2, 4, 8})
+        h->grid[nt] = std::max(1, std::min(dev.num_sms, std::min(E, nt * top_k) * n_chunks));
     *out = h;
     return TS_OK;
 }

@@ -1,295 +1,526 @@
 // ts_gate_up.cu -- fused gate GEMV + ReLU + compaction and gathered up
 // projection + dReLU product + second compaction (Eq. 1 with Eq. 2).
 //
-// Work item = (expert, chunk of kChunk consecutive rows of the row space).
-// One warp owns an item end to end, so no block-level barrier sits in the
-// streaming loop:
-//   1. g = W_gate[j] . x for the chunk's rows and every token of the item;
-//   2. ballot(any token has g > 0) -> the chunk's gate-active rows;
-//   3. u = W_up[j] . x only for those rows (the W_up bytes the method saves);
-//   4. ballot(g > 0 and u > 0) per token -> one bitmap byte per chunk per
-//      token plus the union byte, and c = w_route * g * u for union rows.
-// Rows stream with 16-byte ld.global.nc.L1::no_allocate loads, R rows at a
-// time so each activation element read from shared memory feeds R rows.
-// The activations sit in shared memory as fp32 (the bf16 values exactly).
+// Persistent kernel, one CTA per SM: a producer warp and C consumer
+// warps around a ring of S whole-row slots in shared memory.
+//   * Work item = (expert, chunk of kChunk consecutive rows of the row space);
+//     each CTA owns a contiguous range of items.
+//   * A task is one row in one slot. The producer thread fills free slots
+//     with 1-D bulk copies (cp.async.bulk, 8 KB per row at d=4096 bf16)
+//     completing on the slot's "full" mbarrier. Order: the gate rows of chunk
+//     c, then the up rows of chunk c-kLookahead -- those whose gate
+//     pre-activation is positive for some token, known once that chunk's gate
+//     rows are done. So W_up bytes are read only for gate-active neurons while
+//     the ring stays full.
+//   * Consumer warps take tasks round-robin, dot the slot's row with the
+//     activations (fp32 in shared memory, permuted so 16-byte reads are
+//     conflict-free), release the slot, and record g or u in the chunk's
+//     window state. Each consumer owns two or more slots, so one is in
+//     flight while its owner computes on another. The warp that completes a
+//     chunk's gate rows publishes its gate-active mask to the producer; the warp that completes its up rows
+//     writes the chunk's per-token bitmap bytes, union bytes and
+//     c = w_route * g * u, then frees the window slot.
+//   * In detected mode for a single FFN the producer needs nothing from earlier
+//     kernels, so it starts streaming W_gate before griddepcontrol.wait; the
+//     consumers wait before reading the activations.
+// Every mbarrier wait is bounded (kWaitLimitNs); on expiry the status word
+// gets kStatusTimeout and the CTA drains its copies and returns.
 #include "ts_kernels.cuh"
 
 namespace tsffn {
 
-// Rows per dot-product group and 16-byte loads per lane per row per step,
-// chosen so a warp keeps about 8 KB of weights in flight and the
-// accumulators stay in registers.
-template <typename T, int NT>
-struct GateUpShape {
-    static constexpr int R = NT == 1 ? 1 : (NT == 2 ? 4 : (NT == 4 ? 2 : 1));
-    static constexpr int U = (sizeof(T) == 2 ? 16 : 8) / R;  // R <= 8, so U >= 1
+// consumer warps per CTA for NT tokens per pass; the ring's slot count is a
+// multiple of it
+template <int NT>
+struct GateUpWarps {
+    static constexpr int C = 8;
+    static constexpr int THREADS = (C + 1) * kWarp;
+};
+constexpr int kMaxConsumers = 16;
+constexpr int kWindow = 8;     // chunks in flight per CTA
+constexpr int kLookahead = 3;  // gate chunks issued ahead of their up rows (< kWindow)
+constexpr int kMaxSlots = 32;
+constexpr int kRingBytes = 128 * 1024;  // ring budget: leaves room for down-projection CTAs
+constexpr int kSmemMargin = 8192;       // static shared memory headroom
+
+enum : int { kTaskGate = 0, kTaskUp = 1, kTaskEnd = 2 };
+
+struct Task {
+    int r;     // row within the chunk
+    int cw;    // window slot of the chunk
+    int kind;  // kTaskGate, kTaskUp, kTaskEnd
+    int pad;
 };
 
-// acc[r][k] = sum_i W[row[r]][i] * xs[xo[k] + i] for k < ntok; rows with
-// row[r] < 0 give 0. Every lane ends with the full sums.
-template <typename T, int NT, int R, int U>
-__device__ __forceinline__ void rows_dot(const T* __restrict__ W, const int (&row)[R], int d,
-                                         const float* __restrict__ xs, const int (&xo)[NT],
-                                         int ntok, int lane, float (&acc)[R][NT]) {
-    constexpr int VEC = Vec<T>::N;
-    constexpr int STEP = kWarp * VEC;
-#pragma unroll
-    for (int r = 0; r < R; ++r)
-#pragma unroll
-        for (int k = 0; k < NT; ++k) acc[r][k] = 0.0f;
+template <int NT>
+struct ChunkState {
+    int e, chunk, n_gate, gate_cnt, up_cnt;
+    unsigned gmask;
+    int jr[kChunk];
+    float g[kChunk][NT];
+    float u[kChunk][NT];
+};
 
-    for (int base = lane * VEC; base < d; base += STEP * U) {
-        uint4 v[R][U];
+template <int NT>
+struct GateUpShared {
+    uint64_t full[kMaxSlots];
+    uint64_t empty[kMaxSlots];
+    uint64_t gate_ready[kWindow];
+    uint64_t chunk_free[kWindow];
+    Task task[kMaxSlots];
+    ChunkState<NT> cs[kWindow];
+    ExpertSets es;
+    float red[kMaxConsumers];
+};
+
+struct GateUpCfg {
+    int slots;       // ring slots S
+    int slot_bytes;  // bytes per slot: one row, rounded up to 128
+    int xs_stride;   // floats per activation row in shared memory (d rounded up to 256)
+};
+
+// Activation layout in shared memory: for bf16 rows each 256-element block is
+// stored as [half h][lane l][4] for element l*8 + h*4 + q, so the two 16-byte
+// reads of a lane hit consecutive addresses across the warp.
+template <typename T>
+__device__ __forceinline__ int xs_index(int i) {
+    if (Vec<T>::N == 8)
+        return (i & ~255) | (((i >> 2) & 1) << 7) | (((i >> 3) & 31) << 2) | (i & 3);
+    return i;
+}
+
+// acc[k] = sum_i row[i] * x_{xt[k]}[i] for k < ntok (row in shared memory).
+// Each lane keeps ACC independent partial sums per token (element q of a
+// 16-byte vector goes to sum q % ACC) so the FMAs do not form one serial
+// dependency chain; the sums are combined before the warp reduction.
+template <typename T, int NT>
+__device__ __forceinline__ void smem_row_dot(const unsigned char* row, const float* xs, int xs_stride,
+                                             const int (&xt)[NT], int ntok, int d, int lane,
+                                             float (&acc)[NT]) {
+    constexpr int VEC = Vec<T>::N;
+    constexpr int BLK = kWarp * VEC;
+    constexpr int ACC = NT >= 8 ? 1 : (NT == 4 ? 2 : (NT == 2 ? 4 : VEC));
+    float part[NT][ACC];
+    const float* xr[NT];
 #pragma unroll
-        for (int r = 0; r < R; ++r)
+    for (int k = 0; k < NT; ++k) {
+        xr[k] = xs + (size_t)xt[k] * xs_stride + (VEC == 8 ? lane * 4 : 0);
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const int col = base + u * STEP;
-                if (row[r] >= 0 && col < d)
-                    v[r][u] = ld_stream(W + (size_t)row[r] * (size_t)d + col);
-                else
-                    v[r][u] = make_uint4(0u, 0u, 0u, 0u);
-            }
+        for (int q = 0; q < ACC; ++q) part[k][q] = 0.0f;
+    }
+#pragma unroll 4
+    for (int col = lane * VEC; col < d; col += BLK) {
+        float f[VEC];
+        Vec<T>::unpack(lds128(row + (size_t)col * sizeof(T)), f);
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int col = base + u * STEP;
-            if (col < d) {
-                float f[R][VEC];
-#pragma unroll
-                for (int r = 0; r < R; ++r) Vec<T>::unpack(v[r][u], f[r]);
-#pragma unroll
-                for (int k = 0; k < NT; ++k) {
-                    if (k < ntok) {
-#pragma unroll
-                        for (int q = 0; q < VEC; q += 4) {
-                            const float4 xv = *reinterpret_cast<const float4*>(xs + xo[k] + col + q);
-#pragma unroll
-                            for (int r = 0; r < R; ++r) {
-                                float a = acc[r][k];
-                                a = fmaf(f[r][q + 0], xv.x, a);
-                                a = fmaf(f[r][q + 1], xv.y, a);
-                                a = fmaf(f[r][q + 2], xv.z, a);
-                                a = fmaf(f[r][q + 3], xv.w, a);
-                                acc[r][k] = a;
-                            }
-                        }
-                    }
+        for (int k = 0; k < NT; ++k) {
+            if (NT == 1 || k < ntok) {
+                const float* xk = xr[k];
+                float xv[VEC];
+                if (VEC == 8) {
+                    const int xb = col & ~(BLK - 1);
+                    const uint4 x0 = lds128(xk + xb);
+                    const uint4 x1 = lds128(xk + xb + 128);
+                    xv[0] = __uint_as_float(x0.x); xv[1] = __uint_as_float(x0.y);
+                    xv[2] = __uint_as_float(x0.z); xv[3] = __uint_as_float(x0.w);
+                    xv[4 % VEC] = __uint_as_float(x1.x); xv[5 % VEC] = __uint_as_float(x1.y);
+                    xv[6 % VEC] = __uint_as_float(x1.z); xv[7 % VEC] = __uint_as_float(x1.w);
+                } else {
+                    const uint4 x0 = lds128(xk + col);
+                    xv[0] = __uint_as_float(x0.x); xv[1] = __uint_as_float(x0.y);
+                    xv[2 % VEC] = __uint_as_float(x0.z); xv[3 % VEC] = __uint_as_float(x0.w);
                 }
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) part[k][q % ACC] = fmaf(f[q], xv[q], part[k][q % ACC]);
             }
         }
     }
 #pragma unroll
-    for (int r = 0; r < R; ++r)
+    for (int k = 0; k < NT; ++k) {
+        float s = 0.0f;
 #pragma unroll
-        for (int k = 0; k < NT; ++k) acc[r][k] = warp_sum(acc[r][k]);
+        for (int q = 0; q < ACC; ++q) s += part[k][q];
+        acc[k] = warp_sum(s);
+    }
+}
+
+// Warp-wide: lane 0 waits on `bar`, every lane learns the outcome.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, unsigned parity, int lane, unsigned* status) {
+    int ok = 1;
+    if (lane == 0) {
+        ok = mbar_wait(bar, parity) ? 1 : 0;
+        if (!ok) atomicOr(status, kStatusTimeout);
+    }
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
+// Write a finished chunk's outputs (warp-wide) and free its window slot:
+// per-token gate/both bitmap bytes, union bytes, and c by batch slot.
+template <int NT>
+__device__ void finalize_chunk(const FfnLaunch& a, GateUpShared<NT>& sh, int cw, int lane) {
+    volatile ChunkState<NT>& s = sh.cs[cw];
+    const int e = s.e;
+    const int chunk = s.chunk;
+    const int ntok = sh.es.ntok[e];
+    const unsigned gm = s.gmask;
+    const int j = lane < kChunk ? s.jr[lane] : -1;
+    const bool up_row = lane < kChunk && ((gm >> lane) & 1u);
+    float g[NT], u[NT];
+#pragma unroll
+    for (int k = 0; k < NT; ++k) {
+        g[k] = lane < kChunk ? s.g[lane][k] : 0.0f;
+        u[k] = up_row ? s.u[lane][k] : 0.0f;
+    }
+    unsigned ub = 0u;
+    uint8_t* gb = a.gbits + (size_t)e * a.bits_expert_stride + chunk;
+    uint8_t* bb = a.bbits + (size_t)e * a.bits_expert_stride + chunk;
+    bool both[NT];
+#pragma unroll
+    for (int k = 0; k < NT; ++k) {
+        const bool gk = j >= 0 && g[k] > 0.0f;
+        both[k] = gk && up_row && u[k] > 0.0f;
+        if (k < ntok) {
+            const unsigned gbyte = __ballot_sync(0xffffffffu, gk) & 0xffu;
+            const unsigned bbyte = __ballot_sync(0xffffffffu, both[k]) & 0xffu;
+            ub |= bbyte;
+            if (lane == 0) {
+                const size_t tb = (size_t)(a.bits_tok_base + k) * a.nbytes;
+                gb[tb] = (uint8_t)gbyte;
+                bb[tb] = (uint8_t)bbyte;
+            }
+        }
+    }
+    if (lane == 0) {
+        a.ubits[(size_t)e * a.nbytes + chunk] = (uint8_t)ub;
+        a.ugbits[(size_t)e * a.nbytes + chunk] = (uint8_t)gm;
+    }
+    // c by batch slot: the pass-local token (single FFN) or the global token
+    // (MoE, 0 for tokens not routed to this expert)
+    if (lane < kChunk && ((ub >> lane) & 1u)) {
+        float* cv = a.cval + ((size_t)e * kMaxPass) * a.cval_tok_stride + (size_t)chunk * kChunk + lane;
+        float val[NT];
+#pragma unroll
+        for (int k = 0; k < NT; ++k) val[k] = (k < ntok && both[k]) ? sh.es.w[e][k] * (g[k] * u[k]) : 0.0f;
+        if (a.route == nullptr) {
+#pragma unroll
+            for (int k = 0; k < NT; ++k)
+                if (k < ntok) cv[(size_t)k * a.cval_tok_stride] = val[k];
+        } else {
+            for (int t = 0; t < a.batch; ++t) {
+                float v = 0.0f;
+#pragma unroll
+                for (int k = 0; k < NT; ++k)
+                    if (k < ntok && sh.es.tok[e][k] == t) v = val[k];
+                cv[(size_t)t * a.cval_tok_stride] = v;
+            }
+        }
+    }
+    __syncwarp();
+    __threadfence_block();
+    if (lane == 0) mbar_arrive(&sh.chunk_free[cw]);
+}
+
+// Single-thread wait that records a timeout in the status word.
+__device__ __forceinline__ bool wait_or_flag(uint64_t* bar, unsigned parity, unsigned* status) {
+    if (mbar_wait(bar, parity)) return true;
+    atomicOr(status, kStatusTimeout);
+    return false;
+}
+
+// The producer: one thread (lane 0 of warp 0) issuing row copies in task order.
+template <typename T, int NT>
+__device__ void produce(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char* ring,
+                        const GateUpCfg& cfg, int i0, int i1, int n_chunks) {
+    const unsigned S = (unsigned)cfg.slots;
+    const unsigned row_bytes = (unsigned)(a.d * sizeof(T));
+    const size_t row_elems = (size_t)a.d;
+    unsigned slot = 0, phase = 0, issued = 0;  // next slot, its use parity, tasks issued
+    bool ok = true;
+
+    // One task: row j of matrix w, for row r of the chunk in window slot cw.
+    auto emit = [&](int kind, int cw, int r, int j, const T* w) {
+        if (!wait_or_flag(&sh.empty[slot], phase ^ 1u, a.status)) {
+            ok = false;
+            return;
+        }
+        sh.task[slot] = Task{r, cw, kind, 0};
+        if (kind == kTaskEnd) {
+            mbar_arrive(&sh.full[slot]);
+        } else {
+            mbar_arrive_expect_tx(&sh.full[slot], row_bytes);
+            tma_load_1d(ring + (size_t)slot * cfg.slot_bytes, w + (size_t)j * row_elems, row_bytes,
+                        &sh.full[slot]);
+        }
+        ++issued;
+        if (++slot == S) {
+            slot = 0;
+            phase ^= 1u;
+        }
+    };
+
+    const int n_local = i1 - i0;
+    int jr_hist[kWindow][kChunk];  // the producer's own copy of each window chunk's rows
+    for (int c = 0; ok && c < n_local + kLookahead; ++c) {
+        if (c < n_local) {
+            const int cw = c % kWindow;
+            ok = wait_or_flag(&sh.chunk_free[cw], ((unsigned)(c / kWindow) & 1u) ^ 1u, a.status);
+            if (!ok) break;
+            const int item = i0 + c;
+            const int ea = item / n_chunks;
+            const int chunk = item - ea * n_chunks;
+            const int e = sh.es.act[ea];
+            volatile ChunkState<NT>& s = sh.cs[cw];
+            int* jr = jr_hist[cw];
+            int n_gate = 0;
+#pragma unroll
+            for (int r = 0; r < kChunk; ++r) {
+                const int p = chunk * kChunk + r;
+                int j = -1;
+                if (p < a.n_rows) {
+                    if (a.rows != nullptr) {
+                        const int jj = a.rows[p];
+                        if ((unsigned)jj < (unsigned)a.m && (p == 0 || a.rows[p - 1] < jj))
+                            j = jj;
+                        else
+                            atomicOr(a.status, kStatusBadIndex);
+                    } else {
+                        j = p;
+                    }
+                }
+                jr[r] = j;
+                s.jr[r] = j;
+                n_gate += j >= 0;
+            }
+            s.e = e;
+            s.chunk = chunk;
+            s.n_gate = n_gate;
+            s.gate_cnt = 0;
+            s.up_cnt = 0;
+            s.gmask = 0u;
+            if (n_gate == 0) {
+                // nothing to compute: the chunk's bytes are zero, no c values
+                const int ntok = sh.es.ntok[e];
+                for (int k = 0; k < ntok; ++k) {
+                    const size_t tb = (size_t)(a.bits_tok_base + k) * a.nbytes;
+                    a.gbits[(size_t)e * a.bits_expert_stride + chunk + tb] = 0;
+                    a.bbits[(size_t)e * a.bits_expert_stride + chunk + tb] = 0;
+                }
+                a.ubits[(size_t)e * a.nbytes + chunk] = 0;
+                a.ugbits[(size_t)e * a.nbytes + chunk] = 0;
+                mbar_arrive(&sh.chunk_free[cw]);
+                mbar_arrive(&sh.gate_ready[cw]);
+            } else {
+                const T* wg = static_cast<const T*>(a.ex[e].wg);
+                for (int r = 0; r < kChunk && ok; ++r)
+                    if (jr[r] >= 0) emit(kTaskGate, cw, r, jr[r], wg);
+            }
+        }
+        if (ok && c >= kLookahead) {
+            const int cp = c - kLookahead;
+            const int cw = cp % kWindow;
+            ok = wait_or_flag(&sh.gate_ready[cw], (unsigned)(cp / kWindow) & 1u, a.status);
+            if (!ok) break;
+            volatile ChunkState<NT>& s = sh.cs[cw];
+            const unsigned gm = s.gmask;
+            const T* wu = static_cast<const T*>(a.ex[s.e].wu);
+            const int* jr = jr_hist[cw];
+            for (unsigned m = gm; m && ok; m &= m - 1u) {
+                const int r = __ffs(m) - 1;
+                emit(kTaskUp, cw, r, jr[r], wu);
+            }
+        }
+    }
+    for (int w = 0; w < GateUpWarps<NT>::C && ok; ++w) emit(kTaskEnd, 0, 0, 0, nullptr);
+    // copies in flight must land before the CTA exits: wait on the last use of every slot
+    for (unsigned q = 0; q < S && q < issued; ++q) {
+        slot = slot == 0 ? S - 1 : slot - 1;
+        if (slot == S - 1) phase ^= 1u;
+        if (!wait_or_flag(&sh.full[slot], phase, a.status)) break;
+    }
 }
 
 template <typename T, int NT>
-__global__ void __launch_bounds__(kGateUpWarps * kWarp, 2)
-k_gate_up(const FfnLaunch a, int prefetch_rows) {
-    using S = GateUpShape<T, NT>;
-    constexpr int R = S::R;
-    constexpr int U = S::U;
-    extern __shared__ __align__(16) float xs[];  // [tokens][d] fp32
-    __shared__ ExpertSets es;
-    __shared__ float red[kGateUpWarps];
+__device__ void consume(const FfnLaunch& a, GateUpShared<NT>& sh, const unsigned char* ring,
+                        const float* xs, const GateUpCfg& cfg, int cidx, int lane) {
+    const unsigned S = (unsigned)cfg.slots;
+    constexpr int C = GateUpWarps<NT>::C;
+    // consumer cidx owns slots cidx, cidx + C, ... (S is a multiple of C)
+    unsigned slot = (unsigned)cidx, phase = 0;
+    for (;;) {
+        if (!warp_wait(&sh.full[slot], phase, lane, a.status)) return;
+        const Task tk = sh.task[slot];
+        if (tk.kind == kTaskEnd) return;
+        volatile ChunkState<NT>& s = sh.cs[tk.cw];
+        const int e = s.e;
+        const int ntok = sh.es.ntok[e];
+        int xt[NT];
+#pragma unroll
+        for (int k = 0; k < NT; ++k) xt[k] = k < ntok ? (a.route ? sh.es.tok[e][k] : k) : 0;
+        float acc[NT];
+        smem_row_dot<T, NT>(ring + (size_t)slot * cfg.slot_bytes, xs, cfg.xs_stride, xt, ntok, a.d, lane,
+                            acc);
+        __syncwarp();
+        if (lane == 0) {
+            mbar_arrive(&sh.empty[slot]);
+            volatile float* dst = tk.kind == kTaskGate ? s.g[tk.r] : s.u[tk.r];
+#pragma unroll
+            for (int k = 0; k < NT; ++k) dst[k] = acc[k];
+        }
+        slot += C;
+        if (slot >= S) {
+            slot -= S;
+            phase ^= 1u;
+        }
+        __threadfence_block();
+        int last = 0;
+        if (lane == 0) {
+            if (tk.kind == kTaskGate)
+                last = atomicAdd((int*)&s.gate_cnt, 1) + 1 == s.n_gate;
+            else
+                last = atomicAdd((int*)&s.up_cnt, 1) + 1 == __popc(s.gmask);
+        }
+        last = __shfl_sync(0xffffffffu, last, 0);
+        if (!last) continue;
+        __threadfence_block();
+        if (tk.kind == kTaskGate) {
+            // every gate row of the chunk is in: which rows need their W_up row?
+            bool ga = false;
+            if (lane < kChunk && s.jr[lane] >= 0) {
+#pragma unroll
+                for (int k = 0; k < NT; ++k) ga |= (k < ntok) && (s.g[lane][k] > 0.0f);
+            }
+            const unsigned gm = __ballot_sync(0xffffffffu, ga);
+            if (lane == 0) s.gmask = gm;
+            __syncwarp();
+            __threadfence_block();
+            if (gm == 0u) finalize_chunk<NT>(a, sh, tk.cw, lane);
+            if (lane == 0) mbar_arrive(&sh.gate_ready[tk.cw]);
+        } else {
+            finalize_chunk<NT>(a, sh, tk.cw, lane);
+        }
+    }
+}
+
+template <typename T, int NT>
+__global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up(const FfnLaunch a, const GateUpCfg cfg) {
+    __shared__ GateUpShared<NT> sh;
+    extern __shared__ __align__(128) unsigned char dyn[];
+    float* xs = reinterpret_cast<float*>(dyn);  // [tokens][xs_stride]
+    const int n_x = a.route ? a.batch : a.nt;
+    unsigned char* ring = dyn + (size_t)n_x * cfg.xs_stride * sizeof(float);
 
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
-    const int d = a.d;
-    const int n_chunks = (a.n_rows + kChunk - 1) / kChunk;
-    const int gwarp = blockIdx.x * kGateUpWarps + warp;
-    const int nwarps = gridDim.x * kGateUpWarps;
-
-    // Weights never change, so their first rows may be pulled into L2 while
-    // the previous kernel on the stream is still finishing.
-    if (a.rows == nullptr && a.route == nullptr && gwarp < n_chunks && lane < prefetch_rows) {
-        const int p = gwarp * kChunk + lane;
-        if (p < a.n_rows)
-            prefetch_l2_bulk(static_cast<const T*>(a.ex[0].wg) + (size_t)p * d,
-                             (unsigned)(d * sizeof(T)));
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < cfg.slots; ++s) {
+            mbar_init(&sh.full[s], 1);
+            mbar_init(&sh.empty[s], 1);
+        }
+        for (int w = 0; w < kWindow; ++w) {
+            mbar_init(&sh.gate_ready[w], 1);
+            mbar_init(&sh.chunk_free[w], 1);
+        }
+        mbar_fence_init();
     }
-    pdl_wait();
+    // Single FFN in detected mode: nothing the producer reads comes from an
+    // earlier kernel, so only the consumers wait for it (below).
+    const bool early = a.rows == nullptr && a.route == nullptr;
+    if (!early) pdl_wait();
+    resolve_experts(a, sh.es);  // ends with __syncthreads (barrier init visible)
     pdl_launch_dependents();
 
-    resolve_experts(a, es);
-    const int n_x = a.route ? a.batch : a.nt;
+    const int n_chunks = (a.n_rows + kChunk - 1) / kChunk;
+    const int n_items = sh.es.n_act * n_chunks;
+    const int i0 = (int)((long long)n_items * blockIdx.x / gridDim.x);
+    const int i1 = (int)((long long)n_items * (blockIdx.x + 1) / gridDim.x);
+
+    if (warp == 0) {
+        if (lane == 0) produce<T, NT>(a, sh, ring, cfg, i0, i1, n_chunks);
+        return;
+    }
+    // consumers: activations into shared memory (after the previous kernel)
+    if (early) pdl_wait();
+    const int ctid = threadIdx.x - kWarp;
+    const int cthreads = GateUpWarps<NT>::C * kWarp;
     const int x_tok0 = a.route ? 0 : a.tok0;
     for (int t = 0; t < n_x; ++t) {
+        float* xrow = xs + (size_t)t * cfg.xs_stride;
         if (a.norm_from_h) {
-            block_rmsnorm<T>(a.h + (size_t)(x_tok0 + t) * d, d, xs + (size_t)t * d, red);
+            const float* hr = a.h + (size_t)(x_tok0 + t) * a.d;
+            float ss = 0.0f;
+            for (int i = ctid; i < a.d; i += cthreads) ss = fmaf(hr[i], hr[i], ss);
+            ss = warp_sum(ss);
+            if (lane == 0) sh.red[warp - 1] = ss;
+            named_bar_sync(1, cthreads);
+            float tot = 0.0f;
+            for (int w = 0; w < GateUpWarps<NT>::C; ++w) tot += sh.red[w];
+            const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)a.d), 1e-5f));
+            for (int i = ctid; i < a.d; i += cthreads)
+                xrow[xs_index<T>(i)] = (i == a.d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hr[i], rms));
+            named_bar_sync(1, cthreads);
         } else {
-            for (int i = threadIdx.x; i < d; i += blockDim.x)
-                xs[(size_t)t * d + i] = Vec<T>::load1(a.x, (size_t)(x_tok0 + t) * d + i);
+            for (int i = ctid; i < a.d; i += cthreads)
+                xrow[xs_index<T>(i)] = Vec<T>::load1(a.x, (size_t)(x_tok0 + t) * a.d + i);
         }
     }
-    __syncthreads();
-
-    const int n_items = es.n_act * n_chunks;
-    for (int item = gwarp; item < n_items; item += nwarps) {
-        const int ea = item / n_chunks;
-        const int chunk = item - ea * n_chunks;
-        const int e = es.act[ea];
-        const int ntok = es.ntok[e];
-        const T* __restrict__ wg = static_cast<const T*>(a.ex[e].wg);
-        const T* __restrict__ wu = static_cast<const T*>(a.ex[e].wu);
-        int xo[NT];
-#pragma unroll
-        for (int k = 0; k < NT; ++k) {
-            const int t = k < ntok ? (a.route ? es.tok[e][k] : k) : 0;
-            xo[k] = t * d;
-        }
-
-        // lane r < kChunk: neuron id of row position p0 + r (-1: none)
-        const int p0 = chunk * kChunk;
-        int jr = -1;
-        if (lane < kChunk && p0 + lane < a.n_rows) {
-            const int p = p0 + lane;
-            if (a.rows != nullptr) {
-                const int j = a.rows[p];
-                const bool ok = (unsigned)j < (unsigned)a.m && (p == 0 || a.rows[p - 1] < j);
-                if (ok)
-                    jr = j;
-                else
-                    atomicOr(a.status, kStatusBadIndex);
-            } else {
-                jr = p;
-            }
-        }
-
-        // 1. gate pre-activations of the chunk's rows
-        float greg[NT];
-#pragma unroll
-        for (int k = 0; k < NT; ++k) greg[k] = 0.0f;
-#pragma unroll
-        for (int g0 = 0; g0 < kChunk; g0 += R) {
-            int row[R];
-#pragma unroll
-            for (int r = 0; r < R; ++r) row[r] = __shfl_sync(0xffffffffu, jr, g0 + r);
-            float acc[R][NT];
-            rows_dot<T, NT, R, U>(wg, row, d, xs, xo, ntok, lane, acc);
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-                if (lane == g0 + r)
-#pragma unroll
-                    for (int k = 0; k < NT; ++k) greg[k] = acc[r][k];
-        }
-
-        // 2. gate-active rows: any token with g > 0
-        bool ga = false;
-#pragma unroll
-        for (int k = 0; k < NT; ++k) ga |= (k < ntok) && (greg[k] > 0.0f);
-        ga = ga && jr >= 0;
-        const unsigned gm = __ballot_sync(0xffffffffu, ga);
-
-        // 3. up pre-activations, gathered over the gate-active rows only
-        float ureg[NT];
-#pragma unroll
-        for (int k = 0; k < NT; ++k) ureg[k] = 0.0f;
-        unsigned rest = gm;
-        while (rest) {
-            int row[R];
-            int slot[R];
-#pragma unroll
-            for (int r = 0; r < R; ++r) {
-                if (rest) {
-                    const int b = __ffs(rest) - 1;
-                    rest &= rest - 1u;
-                    slot[r] = b;
-                    row[r] = __shfl_sync(0xffffffffu, jr, b);
-                } else {
-                    slot[r] = -1;
-                    row[r] = -1;
-                }
-            }
-            float acc[R][NT];
-            rows_dot<T, NT, R, U>(wu, row, d, xs, xo, ntok, lane, acc);
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-                if (lane == slot[r])
-#pragma unroll
-                    for (int k = 0; k < NT; ++k) ureg[k] = acc[r][k];
-        }
-
-        // 4. per-token masks, union byte, and c = w * g * u for union rows
-        const bool mine = ga;  // lane's row is gate-active for some token
-        unsigned ub = 0u;
-        uint8_t* gb = a.gbits + (size_t)e * a.bits_expert_stride + chunk;
-        uint8_t* bb = a.bbits + (size_t)e * a.bits_expert_stride + chunk;
-#pragma unroll
-        for (int k = 0; k < NT; ++k) {
-            if (k < ntok) {
-                const bool gk = jr >= 0 && greg[k] > 0.0f;
-                const bool bk = mine && gk && ureg[k] > 0.0f;
-                const unsigned gbyte = __ballot_sync(0xffffffffu, gk) & 0xffu;
-                const unsigned bbyte = __ballot_sync(0xffffffffu, bk) & 0xffu;
-                ub |= bbyte;
-                if (lane == 0) {
-                    const size_t tb = (size_t)(a.bits_tok_base + k) * a.nbytes;
-                    gb[tb] = (uint8_t)gbyte;
-                    bb[tb] = (uint8_t)bbyte;
-                }
-            }
-        }
-        if (lane == 0) {
-            a.ubits[(size_t)e * a.nbytes + chunk] = (uint8_t)ub;
-            a.ugbits[(size_t)e * a.nbytes + chunk] = (uint8_t)gm;
-        }
-        // c by batch slot: the pass-local token (single FFN) or the global
-        // token (MoE, 0 for tokens not routed to this expert)
-        if (lane < kChunk && ((ub >> lane) & 1u)) {
-            float* cv = a.cval + ((size_t)e * kMaxPass) * a.cval_tok_stride + p0 + lane;
-            float val[NT];
-#pragma unroll
-            for (int k = 0; k < NT; ++k)
-                val[k] = (k < ntok && greg[k] > 0.0f && ureg[k] > 0.0f) ? es.w[e][k] * (greg[k] * ureg[k])
-                                                                         : 0.0f;
-            if (a.route == nullptr) {
-#pragma unroll
-                for (int k = 0; k < NT; ++k)
-                    if (k < ntok) cv[(size_t)k * a.cval_tok_stride] = val[k];
-            } else {
-                for (int t = 0; t < a.batch; ++t) {
-                    float v = 0.0f;
-#pragma unroll
-                    for (int k = 0; k < NT; ++k)
-                        if (k < ntok && es.tok[e][k] == t) v = val[k];
-                    cv[(size_t)t * a.cval_tok_stride] = v;
-                }
-            }
-        }
-    }
+    named_bar_sync(1, cthreads);
+    consume<T, NT>(a, sh, ring, xs, cfg, warp - 1, lane);
 }
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+int gate_up_config(int wdtype, int d, int x_tokens, int optin_smem, int* slots, int* slot_bytes,
+                   int* xs_stride, size_t* smem) {
+    const int consumers = x_tokens <= 2 ? GateUpWarps<1>::C : GateUpWarps<8>::C;
+    const int row = d * (wdtype == 1 ? 2 : 4);
+    *slot_bytes = (row + 127) / 128 * 128;
+    *xs_stride = (d + 255) / 256 * 256;
+    const size_t xs_bytes = (size_t)x_tokens * (*xs_stride) * sizeof(float);
+    const long long avail = (long long)optin_smem - kSmemMargin - (long long)xs_bytes;
+    long long s = avail > 0 ? avail / *slot_bytes : 0;
+    s = s < kRingBytes / *slot_bytes ? s : kRingBytes / *slot_bytes;
+    s = s < kMaxSlots ? s : kMaxSlots;
+    // Consumer c takes tasks c, c+C, ...; with S a multiple of C it also owns
+    // every use of its slots, so it never waits on a slot whose previous phase
+    // belongs to another consumer's unfinished task.
+    *slots = (int)(s / consumers * consumers);
+    *smem = xs_bytes + (size_t)(*slots) * (*slot_bytes);
+    return *slots >= consumers ? 0 : -1;
+}
+
+static int g_optin = 0;
 
 template <typename T, int NT>
 static cudaError_t launch_t(const FfnLaunch& a, int grid, cudaStream_t stream, bool pdl) {
     const int n_x = a.route ? a.batch : a.nt;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(kGateUpWarps * kWarp);
-    cfg.dynamicSmemBytes = (size_t)n_x * a.d * sizeof(float);
-    cfg.stream = stream;
+    GateUpCfg cfg;
+    size_t smem = 0;
+    if (gate_up_config(sizeof(T) == 2 ? 1 : 0, a.d, n_x, g_optin, &cfg.slots, &cfg.slot_bytes,
+                       &cfg.xs_stride, &smem) != 0)
+        return cudaErrorInvalidValue;
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(GateUpWarps<NT>::THREADS);
+    lc.dynamicSmemBytes = smem;
+    lc.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = pdl ? 1 : 0;
-    const int prefetch_rows = 2;
-    return cudaLaunchKernelEx(&cfg, k_gate_up<T, NT>, a, prefetch_rows);
+    lc.attrs = attr;
+    lc.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&lc, k_gate_up<T, NT>, a, cfg);
 }
 
-// Allow the largest dynamic shared memory the device offers (minus the
-// kernel's static shared memory) for every instantiation.
 template <typename T, int NT>
 static cudaError_t prepare_t(int optin) {
-    cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, k_gate_up<T, NT>);
-    if (e != cudaSuccess) return e;
     return cudaFuncSetAttribute(k_gate_up<T, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                optin - (int)fa.sharedSizeBytes);
+                                optin - kSmemMargin);
 }
 
 cudaError_t prepare_gate_up(int optin_smem) {
+    static_assert(sizeof(GateUpShared<8>) < kSmemMargin, "static shared memory exceeds the margin");
+    g_optin = optin_smem;
     cudaError_t e = cudaSuccess;
     if (e == cudaSuccess) e = prepare_t<__nv_bfloat16, 1>(optin_smem);
     if (e == cudaSuccess) e = prepare_t<__nv_bfloat16, 2>(optin_smem);
@@ -320,33 +551,6 @@ cudaError_t launch_gate_up(const FfnLaunch& a, int wdtype, int pass_tokens, int 
         }
     }
     return cudaErrorInvalidValue;
-}
-
-template <typename T, int NT>
-static int occupancy_t(size_t smem) {
-    int nb = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k_gate_up<T, NT>, kGateUpWarps * kWarp,
-                                                      smem) != cudaSuccess)
-        return 1;
-    return nb > 0 ? nb : 1;
-}
-
-int gate_up_blocks_per_sm(int wdtype, int pass_tokens, int x_tokens, int d) {
-    const size_t smem = (size_t)x_tokens * d * sizeof(float);
-    if (wdtype == 1) {
-        switch (pass_tokens) {
-            case 1: return occupancy_t<__nv_bfloat16, 1>(smem);
-            case 2: return occupancy_t<__nv_bfloat16, 2>(smem);
-            case 4: return occupancy_t<__nv_bfloat16, 4>(smem);
-            default: return occupancy_t<__nv_bfloat16, 8>(smem);
-        }
-    }
-    switch (pass_tokens) {
-        case 1: return occupancy_t<float, 1>(smem);
-        case 2: return occupancy_t<float, 2>(smem);
-        case 4: return occupancy_t<float, 4>(smem);
-        default: return occupancy_t<float, 8>(smem);
-    }
 }
 
 }  // namespace tsffn

@@ -16,7 +16,6 @@ constexpr int kMaxMoeBatch = 8; // largest MoE batch
 constexpr int kMaxExperts = 16;
 constexpr int kMaxTopK = 4;
 constexpr int kDownWarps = 8;
-constexpr int kGateUpWarps = 8;
 constexpr int kRouterMaxD = 16384;  // router keeps one fp32 activation row in shared memory
 
 // device status bits (OR-ed into the handle's status word)
@@ -136,12 +135,25 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, unsigned parity) {
         : "memory");
     return ok != 0;
 }
+// As mbar_try_wait, but a waiting thread is suspended (it stops issuing)
+// until the phase completes or about `hint_ns` pass.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, unsigned parity, unsigned hint_ns) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+        : "memory");
+    return ok != 0;
+}
 // Wait for the phase with the given parity to complete, for at most
 // kWaitLimitNs; false on timeout (the caller records it and winds down).
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = global_ns();
-    while (!mbar_try_wait(bar, parity))
+    while (!mbar_try_wait_sleep(bar, parity, 1000000u))
         if (global_ns() - t0 > kWaitLimitNs) return false;
     return true;
 }
@@ -298,6 +310,8 @@ cudaError_t launch_router(const RouterLaunch& a, int wdtype, cudaStream_t stream
 cudaError_t prepare_gate_up(int optin_smem);
 cudaError_t prepare_down();
 cudaError_t prepare_router();
-// Resident gate+up CTAs per SM with `x_tokens` activation rows in shared memory.
-int gate_up_blocks_per_sm(int wdtype, int pass_tokens, int x_tokens, int d);
+// Ring geometry of the gate+up kernel for `x_tokens` activation rows in
+// shared memory; -1 if fewer than 4 row slots fit.
+int gate_up_config(int wdtype, int d, int x_tokens, int optin_smem, int* slots, int* slot_bytes,
+                   int* xs_stride, size_t* smem);
 }  // namespace tsffn
