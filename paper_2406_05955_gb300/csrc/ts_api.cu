@@ -16,6 +16,8 @@ using namespace tsffn;
 namespace {
 
 constexpr size_t kAlign = 256;
+// rows of the next layer's W_gate each gate+up CTA prefetches into L2 (stack mode)
+constexpr int kPrefetchRows = 32;
 
 size_t align_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -207,6 +209,7 @@ FfnLaunch ffn_launch(const ts_ffn* h, int batch, const int32_t* rows, int n_rows
     memset(&a, 0, sizeof a);
     a.d = h->d;
     a.m = h->m;
+    a.elem_bytes = elem_size(h->dt);
     a.rows = rows;
     a.n_rows = rows ? n_rows : h->m;
     a.batch = batch;
@@ -374,6 +377,13 @@ ts_status ts_stack_forward(ts_ffn* const* layers, int n_layers, float* hres, int
         a.h = hres;
         a.norm_from_h = 1;
         a.residual_out = 1;
+        const bool next_dense = l + 1 < n_layers && !(active_idx && active_idx[l + 1]);
+        if (next_dense && batch <= kMaxPass) {
+            a.next_wg = layers[l + 1]->wg;
+            a.next_n_rows = layers[l + 1]->m;
+            a.next_grid = layers[l + 1]->grid[pow2_tokens(std::min(kMaxPass, batch))];
+            a.prefetch_rows = kPrefetchRows;
+        }
         for (int t0 = 0; t0 < batch; t0 += kMaxPass) {
             ts_status st = run_pass(h, a, t0, std::min(kMaxPass, batch - t0), stream, true, true);
             if (st != TS_OK) return st;
@@ -496,6 +506,7 @@ ts_status moe_layer(ts_moe* h, const void* x, float* hres, int batch, float* y, 
     memset(&a, 0, sizeof a);
     a.d = h->d;
     a.m = h->m;
+    a.elem_bytes = elem_size(h->dt);
     a.n_rows = h->m;
     a.rows = nullptr;
     a.batch = batch;

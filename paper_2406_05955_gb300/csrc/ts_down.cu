@@ -6,8 +6,10 @@
 // row (32 bf16 or 16 fp32 columns). Every CTA reads the union bitmap words
 // (expert-major, row order), prefix-sums their popcounts and stages the
 // ordered (expert, row) entries in shared memory. A warp instruction covers
-// 8 entries (4 lanes x 16 bytes per row segment); each warp keeps up to 16
-// such instructions in flight, accumulating c * w in fp32 registers per
+// 8 entries (4 lanes x 16 bytes per row segment); each of the 16 warps keeps
+// up to 12 such instructions in flight (the whole list at batch 1 and ~10%
+// activation, in one round trip; the gate+up kernel has already pulled the
+// rows into L2), accumulating c * w in fp32 registers per
 // batch slot. Rows are reduced across lanes (shuffles) and warps (shared
 // memory) in a fixed order and written straight to y (or added to the
 // residual): no partial buffers, no cross-CTA hand-off, bitwise reproducible.
@@ -21,7 +23,7 @@ constexpr int kRowsPerInst = kWarp / kLanesPerRow;  // 8
 
 template <int NT>
 struct DownShape {
-    static constexpr int U = NT <= 2 ? 16 : (NT == 4 ? 8 : 4);  // row groups in flight per warp
+    static constexpr int U = NT <= 2 ? 12 : (NT == 4 ? 8 : 4);  // row groups in flight per warp
 };
 
 __device__ __forceinline__ unsigned union_word(const FfnLaunch& a, const ExpertSets& es,
@@ -46,6 +48,20 @@ __global__ void __launch_bounds__(kDownWarps * kWarp) k_down(const FfnLaunch a) 
     __shared__ int s_total;
     __shared__ float red[kDownWarps][NT][COLS];
 
+    if (a.next_wg != nullptr && a.prefetch_rows > 0) {
+        // independent of the previous kernel: the next layer's weights
+        const int nc = (a.next_n_rows + kChunk - 1) / kChunk;
+        const unsigned row_bytes = (unsigned)(a.d * sizeof(T));
+        const T* nw = static_cast<const T*>(a.next_wg);
+        for (int b = blockIdx.x; b < a.next_grid; b += gridDim.x) {
+            const int r0 = (int)((long long)nc * b / a.next_grid) * kChunk;
+            const int r1 = min((int)((long long)nc * (b + 1) / a.next_grid) * kChunk, a.next_n_rows);
+            const int rn = min(r1 - r0, a.prefetch_rows);
+            const int r = (int)threadIdx.x * kChunk;
+            if (r < rn)
+                prefetch_l2_bulk(nw + (size_t)(r0 + r) * a.d, (unsigned)min(kChunk, rn - r) * row_bytes);
+        }
+    }
     pdl_wait();
     pdl_launch_dependents();
     resolve_experts(a, es);

@@ -194,6 +194,11 @@ __device__ void finalize_chunk(const FfnLaunch& a, GateUpShared<NT>& sh, int cw,
         a.ubits[(size_t)e * a.nbytes + chunk] = (uint8_t)ub;
         a.ugbits[(size_t)e * a.nbytes + chunk] = (uint8_t)gm;
     }
+    // The down projection will gather these W_down rows: pull them into L2
+    // now, while HBM is streaming anyway.
+    if (lane < kChunk && ((ub >> lane) & 1u))
+        prefetch_l2_bulk(static_cast<const unsigned char*>(a.ex[e].wd) + (size_t)j * a.d * a.elem_bytes,
+                         (unsigned)(a.d * a.elem_bytes));
     // c by batch slot: the pass-local token (single FFN) or the global token
     // (MoE, 0 for tokens not routed to this expert)
     if (lane < kChunk && ((ub >> lane) & 1u)) {

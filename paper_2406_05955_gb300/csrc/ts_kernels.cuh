@@ -15,7 +15,7 @@ constexpr int kMaxBatch = 64;   // largest dense batch
 constexpr int kMaxMoeBatch = 8; // largest MoE batch
 constexpr int kMaxExperts = 16;
 constexpr int kMaxTopK = 4;
-constexpr int kDownWarps = 8;
+constexpr int kDownWarps = 16;
 constexpr int kRouterMaxD = 16384;  // router keeps one fp32 activation row in shared memory
 
 // device status bits (OR-ed into the handle's status word)
@@ -44,6 +44,7 @@ struct ExpertPtrs {
 // pass's tokens tok0 .. tok0+nt-1 with weight 1.
 struct FfnLaunch {
     int d, m;
+    int elem_bytes;         // bytes per weight element (2 bf16, 4 fp32)
     int n_rows;             // size of the row space: m, or the list length
     const int32_t* rows;    // predictor list (ascending neuron ids) or nullptr
     int batch;              // tokens of the whole call
@@ -68,6 +69,15 @@ struct FfnLaunch {
     uint8_t* ugbits;        // [expert][nbytes] union gate-active
     unsigned* status;
     int residual_out;       // 1: h += y instead of y =
+    // Stack mode: the next layer's W_gate (nullptr: none), its row count and
+    // its gate+up grid. The down-projection CTAs, before waiting for the
+    // gate+up kernel, prefetch into L2 the first prefetch_rows rows each
+    // next-layer gate+up CTA will stream, so HBM keeps working while this
+    // layer's up rows and down projection finish.
+    const void* next_wg;
+    int next_n_rows;
+    int next_grid;
+    int prefetch_rows;
 };
 
 struct RouterLaunch {
