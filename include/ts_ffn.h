@@ -131,6 +131,35 @@ ts_status ts_ffn_get_active(ts_ffn* h, cudaStream_t stream, int token, int32_t* 
 ts_status ts_ffn_get_error(ts_ffn* h, cudaStream_t stream);
 
 /*
+ * One FFN forward with no handle and no device allocation. The paper has no
+ * counterpart: this is a calling convention, not part of the method. It
+ * computes exactly what ts_ffn_forward computes (Eq. 1 + Eq. 2; active_idx
+ * as there, for the predictor-driven mode of Sec. 7) with the same kernels,
+ * for callers that cannot allocate device memory when they run the FFN.
+ *   d, m, wdtype, w_gate, w_up, w_down   as ts_ffn_create (borrowed for the call)
+ *   x, batch, y, stream, active_idx, n_active   as ts_ffn_forward
+ * Scratch: a fixed array of the library's static device memory (~0.8 MB per
+ * device), sized for m <= TS_NOALLOC_MAX_M and batch <= TS_NOALLOC_MAX_BATCH;
+ * larger sizes return TS_ERR_UNSUPPORTED and launch nothing. Nothing is
+ * allocated or freed by this call.
+ * Set-up: the first call on a device (that device current) looks up the
+ * scratch address and sets kernel attributes; make that first call before
+ * any stream capture on the device.
+ * Concurrency: all calls on a device share the one scratch, so calls whose
+ * executions overlap (other streams, unordered host threads) race; the
+ * caller serialises them.
+ * Errors: argument errors as ts_ffn_create / ts_ffn_forward. A device-side
+ * list error (unsorted or out-of-range ids) skips the offending entries but
+ * is not reported by this entry point.
+ */
+#define TS_NOALLOC_MAX_M 16384
+#define TS_NOALLOC_MAX_BATCH 64
+ts_status ts_ffn_forward_noalloc(int d, int m, ts_dtype wdtype, const void* w_gate,
+                                 const void* w_up, const void* w_down, const void* x, int batch,
+                                 float* y, cudaStream_t stream, const int32_t* active_idx,
+                                 int n_active);
+
+/*
  * Top-k MoE layer (Sec. 4; Mixtral: 2 of 8 experts, Sec. 6.2):
  *     r = x W_r^T, pick the top_k largest logits (lower expert index wins a
  *     tie), w = softmax over the picked logits,

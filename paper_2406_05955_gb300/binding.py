@@ -41,6 +41,7 @@ SIGNATURES = {
     "ts_stack_forward": (I, [P, I, P, I, P, P, P]),
     "ts_ffn_get_active": (I, [P, P, I, P, IP, P, IP]),
     "ts_ffn_get_error": (I, [P, P]),
+    "ts_ffn_forward_noalloc": (I, [I, I, I, P, P, P, P, I, P, P, P, I]),
     "ts_moe_create": (I, [PP, I, I, I, I, P, P, I]),
     "ts_moe_destroy": (None, [P]),
     "ts_moe_forward": (I, [P, P, I, P, P]),
@@ -216,6 +217,25 @@ class Ffn:
             self.close()
         except Exception:
             pass
+
+
+def ffn_forward_noalloc(w_gate, w_up, w_down, x, y, active_idx=None, stream=None) -> torch.Tensor:
+    """``ts_ffn_forward_noalloc``: one FFN forward into the caller's ``y`` with
+    the library's static scratch (no handle, no device allocation)."""
+    for t, n in ((w_gate, "w_gate"), (w_up, "w_up"), (w_down, "w_down"), (x, "x"), (y, "y")):
+        _dev(t, n)
+    m, d = w_gate.shape
+    if w_up.shape != (m, d) or w_down.shape != (m, d):
+        raise ValueError("w_gate, w_up, w_down must all be [m][d]")
+    if not (w_gate.dtype == w_up.dtype == w_down.dtype == x.dtype):
+        raise TypeError("weights and x must share one dtype")
+    if x.dim() != 2 or x.shape[1] != d or y.dtype != torch.float32 or tuple(y.shape) != tuple(x.shape):
+        raise ValueError(f"x must be [batch][{d}] and y [batch][{d}] float32")
+    ptr, n = _list(active_idx)
+    _check(lib().ts_ffn_forward_noalloc(int(d), int(m), _dtype_code(w_gate), w_gate.data_ptr(),
+                                        w_up.data_ptr(), w_down.data_ptr(), x.data_ptr(), x.shape[0],
+                                        y.data_ptr(), _stream(stream), ptr, n), "ts_ffn_forward_noalloc")
+    return y
 
 
 def _addr(arr):
