@@ -16,6 +16,7 @@ independent replica on its own GPU (the path has no cross-GPU exchange) and
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -34,6 +35,32 @@ import torch  # noqa: E402
 METRIC = "sparse-FFN decode tokens/s and achieved HBM GB/s vs needed-bytes roofline"
 UNIT = "tokens/s"
 NOMINAL_HBM_GBS = 7900.0
+
+
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one k_gate_up
+# launch on one full-size layer of the batch-1 stack, from the ncu capture
+# summarised in profiles/k_gate_up-k_down-mistral7b-layer-full.md, and the
+# SHA-256 of the kernel sources it was taken on: once they change, the figure
+# no longer describes the kernel and is reported as null.
+NCU_TRAFFIC = {"bytes": 165.41e6,
+               "sources": ("paper_2406_05955_gb300/csrc/ts_gate_up.cu", "paper_2406_05955_gb300/csrc/ts_kernels.cuh"),
+               "sha256": "9d90164aa6d048d3c5feed9a5a7bc4def4982b54a987566d80ed05ee321eb6e5"}
+
+
+def kernel_sources_sha256(paths) -> str:
+    h = hashlib.sha256()
+    for rel in paths:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def ncu_traffic() -> float | None:
+    try:
+        ok = kernel_sources_sha256(NCU_TRAFFIC["sources"]) == NCU_TRAFFIC["sha256"]
+    except OSError:
+        ok = False
+    return NCU_TRAFFIC["bytes"] if ok else None
 
 
 def load_peaks() -> dict:
@@ -340,7 +367,8 @@ def run_ours(args, dist: Dist) -> dict | None:
                                 else "mistral7b-ffn-stack-bf16-b1-act10"),
                    "d": cfg["d"], "m": cfg["m"], "layers": n_layers, "batch": B,
                    "activation": cfg["activation"], "weights_gb": round(3 * cfg["d"] * cfg["m"] * 2 * n_layers / 1e9, 2),
-                   "l2": "no flush: the 11.3 GB of weights streamed per step exceed the 129 MB L2",
+                   "l2": f"no flush: the {3 * cfg['d'] * cfg['m'] * 2 * n_layers / 1e9:.2f} GB of weights "
+                         "streamed per step exceed the 129 MB L2",
                    "parallelism": f"replicas x{dist.world}"},
         "layers_per_s": value * n_layers / B,
         "needed_bytes_roofline": {
@@ -354,7 +382,8 @@ def run_ours(args, dist: Dist) -> dict | None:
         "roofline": {"bound": "hbm", "kernel": "k_gate_up (gate GEMV + gathered up projection)",
                      "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                      "frac": achieved / peaks["hbm_gbs"], "peak_source": peaks["source"],
-                     "traffic": None, "bytes_per_launch": gate_up_bytes,
+                     "traffic": None if predictor or B != 1 else ncu_traffic(),
+                     "bytes_per_launch": gate_up_bytes,
                      "avg_launch_us": t_gate_up * 1e6},
         "e2e": e2e,
         "gpu_launches": 2 * n_layers * args.steps * ((B + 7) // 8),
