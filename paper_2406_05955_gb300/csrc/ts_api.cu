@@ -80,6 +80,7 @@ struct Scratch {
     uint8_t* ubits = nullptr;
     uint8_t* ugbits = nullptr;
     unsigned* status = nullptr;
+    float* partial = nullptr;  // [gate+up CTA][kAccMaxTokens][d]
 };
 
 }  // namespace
@@ -171,7 +172,10 @@ ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void*
     h->wd = w_down;
     h->dev = dev;
     h->nbytes = (m + 31) / 32 * 4;
+    const int n_chunks = (m + kChunk - 1) / kChunk;
+    for (int nt : {1, 2, 4, 8}) h->grid[nt] = std::max(1, std::min(dev.num_sms, n_chunks));
     const size_t o_cval = h->arena.take((size_t)kMaxPass * m * sizeof(float));
+    const size_t o_p = h->arena.take((size_t)h->grid[kAccMaxTokens] * kAccMaxTokens * d * sizeof(float));
     const size_t o_g = h->arena.take((size_t)max_batch * h->nbytes);
     const size_t o_b = h->arena.take((size_t)max_batch * h->nbytes);
     const size_t o_u = h->arena.take((size_t)h->nbytes);
@@ -188,8 +192,7 @@ ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void*
     h->s.ubits = h->arena.at<uint8_t>(o_u);
     h->s.ugbits = h->arena.at<uint8_t>(o_ug);
     h->s.status = h->arena.at<unsigned>(o_s);
-    const int n_chunks = (m + kChunk - 1) / kChunk;
-    for (int nt : {1, 2, 4, 8}) h->grid[nt] = std::max(1, std::min(dev.num_sms, n_chunks));
+    h->s.partial = h->arena.at<float>(o_p);
     *out = h;
     return TS_OK;
 }
@@ -226,6 +229,8 @@ FfnLaunch ffn_launch(const ts_ffn* h, int batch, const int32_t* rows, int n_rows
     a.ubits = h->s.ubits;
     a.ugbits = h->s.ugbits;
     a.status = h->s.status;
+    a.partial = h->s.partial;
+    a.partial_slots = kAccMaxTokens;
     return a;
 }
 
@@ -243,11 +248,14 @@ ts_status run_pass(ts_ffn* h, FfnLaunch a, int tok0, int nt, cudaStream_t stream
     a.nt = nt;
     a.bits_tok_base = tok0;
     const int w = pow2_tokens(nt);
+    a.partial_ctas = h->grid[w];
     if (gate_up) {
         ts_status st = cuda_status(launch_gate_up(a, h->dt, w, h->grid[w], stream, true));
         if (st != TS_OK) return st;
     }
-    if (down) return cuda_status(launch_down(a, h->dt, w, stream, true));
+    if (down)
+        return cuda_status(w <= kAccMaxTokens ? launch_down_reduce(a, w, stream, true)
+                                              : launch_down(a, h->dt, w, stream, true));
     return TS_OK;
 }
 
@@ -448,7 +456,11 @@ ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype 
     h->dev = dev;
     h->nbytes = (h->m + 31) / 32 * 4;
     const int m = h->m, E = n_experts;
+    const int n_chunks = (m + kChunk - 1) / kChunk;
+    for (int nt : {1, 2, 4, 8})
+        h->grid[nt] = std::max(1, std::min(dev.num_sms, std::min(E, nt * top_k) * n_chunks));
     const size_t o_cval = h->arena.take((size_t)E * kMaxPass * m * sizeof(float));
+    const size_t o_p = h->arena.take((size_t)h->grid[kAccMaxTokens] * kAccMaxTokens * d * sizeof(float));
     const size_t o_g = h->arena.take((size_t)E * kMaxPass * h->nbytes);
     const size_t o_b = h->arena.take((size_t)E * kMaxPass * h->nbytes);
     const size_t o_u = h->arena.take((size_t)E * h->nbytes);
@@ -469,9 +481,7 @@ ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype 
     h->s.status = h->arena.at<unsigned>(o_s);
     h->route = h->arena.at<TokenRoute>(o_r);
     h->xbuf = h->arena.at<void>(o_x);
-    const int n_chunks = (m + kChunk - 1) / kChunk;
-    for (int nt : {1, 2, 4, 8})
-        h->grid[nt] = std::max(1, std::min(dev.num_sms, std::min(E, nt * top_k) * n_chunks));
+    h->s.partial = h->arena.at<float>(o_p);
     *out = h;
     return TS_OK;
 }
@@ -532,9 +542,13 @@ ts_status moe_layer(ts_moe* h, const void* x, float* hres, int batch, float* y, 
     a.ugbits = h->s.ugbits;
     a.status = h->s.status;
     const int w = pow2_tokens(batch);
+    a.partial = h->s.partial;
+    a.partial_slots = kAccMaxTokens;
+    a.partial_ctas = h->grid[w];
     st = cuda_status(launch_gate_up(a, h->dt, w, h->grid[w], stream, true));
     if (st != TS_OK) return st;
-    return cuda_status(launch_down(a, h->dt, w, stream, true));
+    return cuda_status(w <= kAccMaxTokens ? launch_down_reduce(a, w, stream, true)
+                                          : launch_down(a, h->dt, w, stream, true));
 }
 
 }  // namespace

@@ -2,7 +2,9 @@
 // (the "Combined(x) W_down" of Eq. 1, restricted to the non-zero dReLU
 // activations of Eq. 2).
 //
-// One CTA per slice of kDownCols output columns: 64 bytes of every active
+// Passes of up to kAccMaxTokens tokens: the gate+up CTAs have already summed
+// their own rows; k_down_reduce (below) adds their partials. Wider passes:
+// k_down gathers the rows itself. One CTA per slice of kDownCols output columns: 64 bytes of every active
 // row (32 bf16 or 16 fp32 columns). Every CTA reads the union bitmap words
 // (expert-major, row order), prefix-sums their popcounts and stages the
 // ordered (expert, row) entries in shared memory. A warp instruction covers
@@ -212,6 +214,110 @@ static cudaError_t launch_t(const FfnLaunch& a, cudaStream_t stream, bool pdl) {
     cfg.attrs = attr;
     cfg.numAttrs = pdl ? 1 : 0;
     return cudaLaunchKernelEx(&cfg, k_down<T, NT>, a);
+}
+
+// ---------------------------------------------------------------------------
+// Passes of <= kAccMaxTokens tokens: every gate+up CTA has already summed
+// c_j W_down[j,:] over its own both-active rows (its accumulator warp) into
+// its block of the partial buffer. Here the blocks are added in CTA order:
+// one CTA per 64 output columns, a half-warp covers them with 16-byte loads,
+// the 32 half-warps take every 32nd block, and the half-warp and warp sums
+// are combined in a fixed order (bitwise reproducible).
+// ---------------------------------------------------------------------------
+constexpr int kRedCols = 64;
+constexpr int kRedThreads = 512;
+constexpr int kRedWarps = kRedThreads / kWarp;
+constexpr int kRedLanes = kRedCols / 4;  // lanes of a half-warp, a float4 each
+
+template <int NT>
+__global__ void __launch_bounds__(kRedThreads) k_down_reduce(const FfnLaunch a) {
+    __shared__ float4 red[kRedWarps][NT][kRedLanes];
+    pdl_wait();
+    pdl_launch_dependents();
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int hw = lane / kRedLanes;
+    const int cl = lane % kRedLanes;
+    const int d = a.d;
+    const int n_slots = a.route ? a.batch : a.nt;
+    const int col = blockIdx.x * kRedCols + cl * 4;
+    const bool valid = col < d;
+
+    // this thread's output (n_slots * kRedCols <= kRedThreads): its residual
+    // is read while the partials load
+    const int out_k = threadIdx.x / kRedCols;
+    const int out_c = blockIdx.x * kRedCols + (threadIdx.x - out_k * kRedCols);
+    const bool has_out = out_k < n_slots && out_c < d;
+    const size_t out_i = (size_t)(a.route ? out_k : a.tok0 + out_k) * d + out_c;
+    float h_old = 0.0f;
+    if (has_out && a.residual_out) h_old = a.h[out_i];
+
+    float4 acc[NT];
+#pragma unroll
+    for (int k = 0; k < NT; ++k) acc[k] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    if (valid) {
+        const size_t cta_stride = (size_t)a.partial_slots * d;
+        for (int b = warp * 2 + hw; b < a.partial_ctas; b += 2 * kRedWarps) {
+            const float* p = a.partial + (size_t)b * cta_stride + col;
+#pragma unroll
+            for (int k = 0; k < NT; ++k)
+                if (k < n_slots) {
+                    const float4 v = *reinterpret_cast<const float4*>(p + (size_t)k * d);
+                    acc[k].x += v.x;
+                    acc[k].y += v.y;
+                    acc[k].z += v.z;
+                    acc[k].w += v.w;
+                }
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < NT; ++k) {
+        // half-warp 0 + half-warp 1: both halves end with the same sum
+        acc[k].x += __shfl_xor_sync(0xffffffffu, acc[k].x, kRedLanes);
+        acc[k].y += __shfl_xor_sync(0xffffffffu, acc[k].y, kRedLanes);
+        acc[k].z += __shfl_xor_sync(0xffffffffu, acc[k].z, kRedLanes);
+        acc[k].w += __shfl_xor_sync(0xffffffffu, acc[k].w, kRedLanes);
+    }
+    if (hw == 0) {
+#pragma unroll
+        for (int k = 0; k < NT; ++k) red[warp][k][cl] = acc[k];
+    }
+    __syncthreads();
+    if (has_out) {
+        const int c = out_c - blockIdx.x * kRedCols;
+        float sum = 0.0f;
+#pragma unroll
+        for (int w = 0; w < kRedWarps; ++w) sum += reinterpret_cast<const float*>(&red[w][out_k][0])[c];
+        if (a.residual_out)
+            a.h[out_i] = h_old + sum;
+        else
+            a.y[out_i] = sum;
+    }
+}
+
+template <int NT>
+static cudaError_t launch_reduce_t(const FfnLaunch& a, cudaStream_t stream, bool pdl) {
+    static_assert(NT * kRedCols <= kRedThreads, "one output per thread");
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((a.d + kRedCols - 1) / kRedCols);
+    cfg.blockDim = dim3(kRedThreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, k_down_reduce<NT>, a);
+}
+
+cudaError_t launch_down_reduce(const FfnLaunch& a, int pass_tokens, cudaStream_t stream, bool pdl) {
+    if (a.partial == nullptr || a.partial_ctas < 1) return cudaErrorInvalidValue;
+    switch (pass_tokens) {
+        case 1: return launch_reduce_t<1>(a, stream, pdl);
+        case 2: return launch_reduce_t<2>(a, stream, pdl);
+    }
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t prepare_down() { return cudaSuccess; }

@@ -23,8 +23,14 @@
 //   * In detected mode for a single FFN the producer needs nothing from earlier
 //     kernels, so it starts streaming W_gate before griddepcontrol.wait; the
 //     consumers wait before reading the activations.
+//   * Passes of up to kAccMaxTokens tokens also do this CTA's share of the
+//     down projection at the end (down_partial): the CTA's W_down rows are
+//     staged in the idle ring and summed into its block of the partial
+//     buffer, which the down kernel's reduction adds up over the CTAs.
 // Every mbarrier wait is bounded (kWaitLimitNs); on expiry the status word
 // gets kStatusTimeout and the CTA drains its copies and returns.
+#include <type_traits>
+
 #include "ts_kernels.cuh"
 
 namespace tsffn {
@@ -54,15 +60,30 @@ struct Task {
 
 template <int NT>
 struct ChunkState {
-    int e, chunk, n_gate, gate_cnt, up_cnt;
+    int e, chunk, q, n_gate, gate_cnt, up_cnt;
     unsigned gmask;
     int jr[kChunk];
     float g[kChunk][NT];
     float u[kChunk][NT];
 };
 
+// Passes of <= kAccMaxTokens tokens: what the end-of-CTA down projection
+// needs from each finished chunk (local index q < kMaxLocal; later chunks are
+// read back from global memory), and the staging of its W_down rows.
+constexpr int kMaxLocal = 32;
+struct PartialShared {
+    uint8_t ub[kMaxLocal];                         // both-active rows of chunk q
+    float c[kMaxLocal][kChunk][kAccMaxTokens];     // their c values by batch slot
+    int2 meta[kMaxSlots];                          // (expert, position) of the row in each slot
+    float cs[kMaxSlots][kAccMaxTokens];            // its c values
+    int n_rows, next_item;                         // rows staged this round, first item of the next
+    uint64_t landed;                               // every staged row is in its slot
+};
+struct NoPartial {};
+
 template <int NT>
 struct GateUpShared {
+    typename std::conditional<(NT <= kAccMaxTokens), PartialShared, NoPartial>::type pd;
     uint64_t full[kMaxSlots];
     uint64_t empty[kMaxSlots];
     uint64_t gate_ready[kWindow];
@@ -220,9 +241,165 @@ __device__ void finalize_chunk(const FfnLaunch& a, GateUpShared<NT>& sh, int cw,
             }
         }
     }
+    if constexpr (NT <= kAccMaxTokens) {
+        const int q = s.q;
+        if (q < kMaxLocal) {
+            if (lane == 0) sh.pd.ub[q] = (uint8_t)ub;
+            if (lane < kChunk) {
+#pragma unroll
+                for (int t = 0; t < kAccMaxTokens; ++t) {
+                    float v = 0.0f;
+#pragma unroll
+                    for (int k = 0; k < NT; ++k) {
+                        const int slot_of_k = a.route ? sh.es.tok[e][k] : k;
+                        if (k < ntok && both[k] && slot_of_k == t) v = sh.es.w[e][k] * (g[k] * u[k]);
+                    }
+                    sh.pd.c[q][lane][t] = v;
+                }
+            }
+        }
+    }
     __syncwarp();
     __threadfence_block();
     if (lane == 0) mbar_arrive(&sh.chunk_free[cw]);
+}
+
+// This CTA's share of the down projection (Eq. 1 over the non-zero
+// activations of Eq. 2), once every chunk of the CTA is finalized: for each
+// batch slot t,
+//     partial[cta][t][:] = sum over the CTA's both-active rows j, in local
+//                          chunk order and row order, of c_{t,j} W_down[j,:].
+// The ring is idle by then: consumer warp 0 stages up to S rows per round in
+// it by bulk copy (the finalizer already pulled them into L2), then every
+// consumer warp adds its column blocks over the staged rows. A round after
+// the first adds onto the stored partial, so the order stays fixed and the
+// result is bitwise reproducible.
+template <typename T, int NT>
+__device__ void down_partial(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char* ring,
+                             const GateUpCfg& cfg, int i0, int i1, int n_chunks, int cidx, int lane) {
+    constexpr int VEC = Vec<T>::N;
+    constexpr int BLK = kWarp * VEC;
+    constexpr int C = GateUpWarps<NT>::C;
+    constexpr int AT = kAccMaxTokens;
+    const int cthreads = C * kWarp;
+    const int d = a.d;
+    const unsigned row_bytes = (unsigned)(d * sizeof(T));
+    const int n_slots = a.route ? a.batch : a.nt;
+    const int S = cfg.slots;
+    float* pbase = a.partial + (size_t)blockIdx.x * a.partial_slots * d;
+    const int nblk = (d + BLK - 1) / BLK;
+    int it = i0;
+    unsigned round = 0;
+    bool ok = true;
+    do {
+        if (cidx == 0) {
+            // stage the rows of the next items, whole items only, at most S rows
+            int n = 0;
+            bool full = false;
+            while (!full && it < i1) {
+                const int item = it + lane;
+                unsigned bits = 0u;
+                int e = 0, chunk = 0;
+                if (item < i1) {
+                    const int ea = item / n_chunks;
+                    chunk = item - ea * n_chunks;
+                    e = sh.es.act[ea];
+                    const int q = item - i0;
+                    bits = q < kMaxLocal ? (unsigned)sh.pd.ub[q]
+                                         : (unsigned)*reinterpret_cast<const volatile uint8_t*>(
+                                               a.ubits + (size_t)e * a.nbytes + chunk);
+                }
+                const int cnt = __popc(bits);
+                int incl = cnt;
+#pragma unroll
+                for (int o = 1; o < kWarp; o <<= 1) {
+                    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += v;
+                }
+                // items that fit this round: a prefix of the lanes
+                const bool fits = item < i1 && n + incl <= S;
+                const unsigned take = __ballot_sync(0xffffffffu, fits);
+                const int n_take = __popc(take);  // lanes 0 .. n_take-1
+                if (fits) {
+                    int pos = n + incl - cnt;
+                    const int q = item - i0;
+                    for (unsigned b = bits; b; b &= b - 1u) {
+                        const int r = __ffs(b) - 1;
+                        const int p = chunk * kChunk + r;
+                        const int j = a.rows ? a.rows[p] : p;
+                        sh.pd.meta[pos] = make_int2(e, p);
+#pragma unroll
+                        for (int t = 0; t < AT; ++t)
+                            sh.pd.cs[pos][t] =
+                                q < kMaxLocal ? sh.pd.c[q][r][t]
+                                              : (t < n_slots ? a.cval[((size_t)e * kMaxPass + t) * a.cval_tok_stride + p]
+                                                             : 0.0f);
+                        mbar_expect_tx(&sh.pd.landed, row_bytes);
+                        tma_load_1d(ring + (size_t)pos * cfg.slot_bytes,
+                                    static_cast<const T*>(a.ex[e].wd) + (size_t)j * d, row_bytes, &sh.pd.landed);
+                        ++pos;
+                    }
+                }
+                const int added = __shfl_sync(0xffffffffu, incl, n_take > 0 ? n_take - 1 : 0);
+                if (n_take > 0) n += added;
+                it += n_take;
+                full = n_take < kWarp && it < i1;  // the next item did not fit
+            }
+            __syncwarp();
+            if (lane == 0) {
+                sh.pd.n_rows = n;
+                sh.pd.next_item = it;
+                mbar_arrive(&sh.pd.landed);  // the phase completes when every copy has landed
+            }
+        }
+        named_bar_sync(1, cthreads);
+        const int n = sh.pd.n_rows;
+        const int next = sh.pd.next_item;
+        int okw = 1;
+        if (lane == 0) {
+            okw = mbar_wait(&sh.pd.landed, round & 1u) ? 1 : 0;
+            if (!okw) atomicOr(a.status, kStatusTimeout);
+        }
+        if (!__shfl_sync(0xffffffffu, okw, 0)) {
+            // copies still in flight must land before the CTA exits
+            ok = false;
+            if (lane == 0) mbar_wait(&sh.pd.landed, round & 1u);
+            __syncwarp();
+        }
+        if (ok) {
+            for (int blk = cidx; blk < nblk; blk += C) {
+                const int col = blk * BLK + lane * VEC;
+                if (col >= d) continue;
+                float acc[AT][VEC];
+#pragma unroll
+                for (int t = 0; t < AT; ++t)
+#pragma unroll
+                    for (int v = 0; v < VEC; ++v)
+                        acc[t][v] = (round > 0 && t < n_slots) ? pbase[(size_t)t * d + col + v] : 0.0f;
+                for (int i = 0; i < n; ++i) {
+                    float f[VEC];
+                    Vec<T>::unpack(lds128(ring + (size_t)i * cfg.slot_bytes + (size_t)col * sizeof(T)), f);
+#pragma unroll
+                    for (int t = 0; t < AT; ++t) {
+                        const float c = sh.pd.cs[i][t];
+#pragma unroll
+                        for (int v = 0; v < VEC; ++v) acc[t][v] = fmaf(c, f[v], acc[t][v]);
+                    }
+                }
+#pragma unroll
+                for (int t = 0; t < AT; ++t)
+                    if (t < n_slots) {
+                        float4* o = reinterpret_cast<float4*>(pbase + (size_t)t * d + col);
+#pragma unroll
+                        for (int v = 0; v < VEC; v += 4)
+                            o[v / 4] = make_float4(acc[t][v], acc[t][v + 1], acc[t][v + 2], acc[t][v + 3]);
+                    }
+            }
+        }
+        it = next;
+        ++round;
+        named_bar_sync(1, cthreads);  // the slots and the list are reused next round
+    } while (ok && it < i1);
 }
 
 // Single-thread wait that records a timeout in the status word.
@@ -298,6 +475,7 @@ __device__ void produce(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char*
             }
             s.e = e;
             s.chunk = chunk;
+            s.q = c;
             s.n_gate = n_gate;
             s.gate_cnt = 0;
             s.up_cnt = 0;
@@ -312,6 +490,9 @@ __device__ void produce(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char*
                 }
                 a.ubits[(size_t)e * a.nbytes + chunk] = 0;
                 a.ugbits[(size_t)e * a.nbytes + chunk] = 0;
+                if constexpr (NT <= kAccMaxTokens) {
+                    if (c < kMaxLocal) sh.pd.ub[c] = 0;
+                }
                 mbar_arrive(&sh.chunk_free[cw]);
                 mbar_arrive(&sh.gate_ready[cw]);
             } else {
@@ -425,6 +606,7 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up(const F
             mbar_init(&sh.gate_ready[w], 1);
             mbar_init(&sh.chunk_free[w], 1);
         }
+        if constexpr (NT <= kAccMaxTokens) mbar_init(&sh.pd.landed, 1);
         mbar_fence_init();
     }
     // Single FFN in detected mode: nothing the producer reads comes from an
@@ -470,6 +652,12 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up(const F
     }
     named_bar_sync(1, cthreads);
     consume<T, NT>(a, sh, ring, xs, cfg, warp - 1, lane);
+    if constexpr (NT <= kAccMaxTokens) {
+        // every chunk is finalized and every ring copy consumed once all
+        // consumers are here
+        named_bar_sync(1, cthreads);
+        down_partial<T, NT>(a, sh, ring, cfg, i0, i1, n_chunks, warp - 1, lane);
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -504,6 +692,8 @@ static cudaError_t launch_t(const FfnLaunch& a, int grid, cudaStream_t stream, b
     if (gate_up_config(sizeof(T) == 2 ? 1 : 0, a.d, n_x, g_optin, &cfg.slots, &cfg.slot_bytes,
                        &cfg.xs_stride, &smem) != 0)
         return cudaErrorInvalidValue;
+    if (NT <= kAccMaxTokens && (a.partial == nullptr || a.partial_slots < n_x || a.partial_ctas < grid))
+        return cudaErrorInvalidValue;
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(grid);
     lc.blockDim = dim3(GateUpWarps<NT>::THREADS);
@@ -524,7 +714,9 @@ static cudaError_t prepare_t(int optin) {
 }
 
 cudaError_t prepare_gate_up(int optin_smem) {
-    static_assert(sizeof(GateUpShared<8>) < kSmemMargin, "static shared memory exceeds the margin");
+    static_assert(sizeof(GateUpShared<8>) < kSmemMargin && sizeof(GateUpShared<4>) < kSmemMargin &&
+                      sizeof(GateUpShared<2>) < kSmemMargin && sizeof(GateUpShared<1>) < kSmemMargin,
+                  "static shared memory exceeds the margin");
     g_optin = optin_smem;
     cudaError_t e = cudaSuccess;
     if (e == cudaSuccess) e = prepare_t<__nv_bfloat16, 1>(optin_smem);

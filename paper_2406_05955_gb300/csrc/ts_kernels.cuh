@@ -16,6 +16,11 @@ constexpr int kMaxMoeBatch = 8; // largest MoE batch
 constexpr int kMaxExperts = 16;
 constexpr int kMaxTopK = 4;
 constexpr int kDownWarps = 16;
+// Passes of at most this many tokens fold the down projection into the
+// gate+up kernel (an accumulator warp per CTA writes a partial y) and finish
+// it with a reduction over the CTAs' partials; wider passes gather W_down rows
+// in a separate kernel.
+constexpr int kAccMaxTokens = 2;
 constexpr int kRouterMaxD = 16384;  // router keeps one fp32 activation row in shared memory
 
 // device status bits (OR-ed into the handle's status word)
@@ -69,6 +74,12 @@ struct FfnLaunch {
     uint8_t* ugbits;        // [expert][nbytes] union gate-active
     unsigned* status;
     int residual_out;       // 1: h += y instead of y =
+    // Partial down projections of passes of <= kAccMaxTokens tokens,
+    // [gate+up CTA][partial_slots][d] fp32: gate+up CTA b writes slots
+    // 0 .. n_slots-1 of block b; the reduction sums blocks 0 .. partial_ctas-1.
+    float* partial;
+    int partial_slots;
+    int partial_ctas;
     // Stack mode: the next layer's W_gate (nullptr: none), its row count and
     // its gate+up grid. The down-projection CTAs, before waiting for the
     // gate+up kernel, prefetch into L2 the first prefetch_rows rows each
@@ -132,6 +143,11 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
 }
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, unsigned bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+// Raise the transaction count the current phase waits for, without arriving.
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, unsigned bytes) {
+    asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
                  : "memory");
 }
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, unsigned parity) {
@@ -315,6 +331,8 @@ cudaError_t launch_gate_up(const FfnLaunch& a, int wdtype, int pass_tokens, int 
                            cudaStream_t stream, bool pdl);
 cudaError_t launch_down(const FfnLaunch& a, int wdtype, int pass_tokens, cudaStream_t stream,
                         bool pdl);
+// Sum of the gate+up CTAs' partial down projections (passes of <= kAccMaxTokens).
+cudaError_t launch_down_reduce(const FfnLaunch& a, int pass_tokens, cudaStream_t stream, bool pdl);
 cudaError_t launch_router(const RouterLaunch& a, int wdtype, cudaStream_t stream, bool pdl);
 // Set per-kernel attributes once per device, before any launch or capture.
 cudaError_t prepare_gate_up(int optin_smem);

@@ -152,7 +152,9 @@ extern "C" ts_status ts_ffn_forward_noalloc(int d, int m, ts_dtype wdtype, const
 
     for (int t0 = 0; t0 < batch; t0 += kMaxPass) {
         const int nt = std::min(kMaxPass, batch - t0);
-        const int w = nt <= 1 ? 1 : nt <= 2 ? 2 : nt <= 4 ? 4 : 8;
+        // widths of at least 4 gather W_down in the down kernel and need no
+        // per-CTA partial buffer
+        const int w = nt <= 4 ? 4 : 8;
         a.tok0 = t0;
         a.nt = nt;
         a.bits_tok_base = t0;
