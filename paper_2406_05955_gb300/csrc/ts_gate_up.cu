@@ -661,6 +661,299 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up(const F
 }
 
 // ---------------------------------------------------------------------------
+// Passes of 4-8 tokens, bf16, d % 256 == 0: tensor-core variant.
+//
+// At these batch sizes the per-row dot products are a skinny GEMM
+// ([tokens x d] x [d x rows]) that CUDA-core FMAs can no longer hide behind
+// HBM. Tasks become groups of up to 8 rows of one chunk (its gate rows, or its
+// gate-active up rows), two groups in flight in a ring of 16 padded row slots.
+// All consumer warps work on each group, warp w over the w-th K slice, with
+// mma.sync m16n8k16 (A = the activations, 8 token rows plus 8 zero rows;
+// B = the 8 weight rows; fp32 accumulation); the slices are added in warp
+// order, so results do not depend on timing. Rows are padded by 16 bytes in
+// shared memory so ldmatrix reads are free of bank conflicts.
+// ---------------------------------------------------------------------------
+constexpr int kMmaGroups = 2;    // groups in flight
+constexpr int kMmaRowPad = 16;   // bytes after every row in shared memory
+constexpr int kMmaDAlign = 256;  // d must be a multiple (even K-step count per warp)
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+// d += A * B for one m16n8k16 step; A rows 8-15 are zero (no token there).
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
+    const uint32_t z = 0u;
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(z), "r"(a2), "r"(z), "r"(b0), "r"(b1));
+}
+
+struct MmaCfg {
+    int row_stride;  // bytes per row in shared memory (d * 2 + kMmaRowPad)
+};
+
+// The producer of the tensor-core variant: groups in task order (gate rows of
+// chunk c, then the up rows of chunk c-1), one expect-tx barrier per group.
+template <int NT>
+__device__ void produce_mma(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char* ring, const MmaCfg& mc,
+                            int i0, int i1, int n_chunks) {
+    using T = __nv_bfloat16;
+    const unsigned row_bytes = (unsigned)(a.d * sizeof(T));
+    unsigned grp = 0;
+    bool ok = true;
+    auto emit = [&](int kind, int cw, const int* jr, unsigned mask, const T* w) {
+        const unsigned g = grp % kMmaGroups;
+        const unsigned ph = (grp / kMmaGroups) & 1u;
+        if (!wait_or_flag(&sh.empty[g], ph ^ 1u, a.status)) {
+            ok = false;
+            return;
+        }
+        sh.task[g] = Task{(int)mask, cw, kind, 0};
+        if (kind == kTaskEnd) {
+            mbar_arrive(&sh.full[g]);
+        } else {
+            mbar_arrive_expect_tx(&sh.full[g], (unsigned)__popc(mask) * row_bytes);
+            for (unsigned m = mask; m; m &= m - 1u) {
+                const int r = __ffs(m) - 1;
+                tma_load_1d(ring + ((size_t)g * kChunk + r) * mc.row_stride, w + (size_t)jr[r] * a.d, row_bytes,
+                            &sh.full[g]);
+            }
+        }
+        ++grp;
+    };
+    const int n_local = i1 - i0;
+    constexpr int L = 1;  // gate groups ahead of their up group
+    int jr_hist[kWindow][kChunk];
+    for (int c = 0; ok && c < n_local + L; ++c) {
+        if (c < n_local) {
+            const int cw = c % kWindow;
+            ok = wait_or_flag(&sh.chunk_free[cw], ((unsigned)(c / kWindow) & 1u) ^ 1u, a.status);
+            if (!ok) break;
+            const int item = i0 + c;
+            const int ea = item / n_chunks;
+            const int chunk = item - ea * n_chunks;
+            const int e = sh.es.act[ea];
+            volatile ChunkState<NT>& s = sh.cs[cw];
+            int* jr = jr_hist[cw];
+            unsigned mask = 0u;
+#pragma unroll
+            for (int r = 0; r < kChunk; ++r) {
+                const int p = chunk * kChunk + r;
+                int j = -1;
+                if (p < a.n_rows) {
+                    if (a.rows != nullptr) {
+                        const int jj = a.rows[p];
+                        if ((unsigned)jj < (unsigned)a.m && (p == 0 || a.rows[p - 1] < jj))
+                            j = jj;
+                        else
+                            atomicOr(a.status, kStatusBadIndex);
+                    } else {
+                        j = p;
+                    }
+                }
+                jr[r] = j;
+                s.jr[r] = j;
+                if (j >= 0) mask |= 1u << r;
+            }
+            s.e = e;
+            s.chunk = chunk;
+            s.q = c;
+            s.n_gate = __popc(mask);
+            s.gate_cnt = 0;
+            s.up_cnt = 0;
+            s.gmask = 0u;
+            if (mask == 0u) {
+                const int ntok = sh.es.ntok[e];
+                for (int k = 0; k < ntok; ++k) {
+                    const size_t tb = (size_t)(a.bits_tok_base + k) * a.nbytes;
+                    a.gbits[(size_t)e * a.bits_expert_stride + chunk + tb] = 0;
+                    a.bbits[(size_t)e * a.bits_expert_stride + chunk + tb] = 0;
+                }
+                a.ubits[(size_t)e * a.nbytes + chunk] = 0;
+                a.ugbits[(size_t)e * a.nbytes + chunk] = 0;
+                mbar_arrive(&sh.chunk_free[cw]);
+                mbar_arrive(&sh.gate_ready[cw]);
+            } else {
+                emit(kTaskGate, cw, jr, mask, static_cast<const T*>(a.ex[e].wg));
+            }
+        }
+        if (ok && c >= L) {
+            const int cp = c - L;
+            const int cw = cp % kWindow;
+            ok = wait_or_flag(&sh.gate_ready[cw], (unsigned)(cp / kWindow) & 1u, a.status);
+            if (!ok) break;
+            volatile ChunkState<NT>& s = sh.cs[cw];
+            const unsigned gm = s.gmask;
+            if (gm) emit(kTaskUp, cw, jr_hist[cw], gm, static_cast<const T*>(a.ex[s.e].wu));
+        }
+    }
+    if (ok) emit(kTaskEnd, 0, nullptr, 0u, nullptr);
+    // copies in flight must land before the CTA exits
+    for (unsigned q = 0; q < kMmaGroups && q < grp; ++q) {
+        const unsigned gi = grp - 1 - q;
+        if (!wait_or_flag(&sh.full[gi % kMmaGroups], (gi / kMmaGroups) & 1u, a.status)) break;
+    }
+}
+
+// The consumers of the tensor-core variant (C warps, all on every group).
+template <int NT>
+__device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsigned char* ring,
+                            const unsigned char* xb, float* red, const MmaCfg& mc, int cidx, int lane) {
+    constexpr int C = GateUpWarps<NT>::C;
+    const int cthreads = C * kWarp;
+    const int n_ks = a.d / 16;          // K steps of 16
+    const int per = n_ks / C;           // even: d % kMmaDAlign == 0
+    const int ks0 = cidx * per;
+    const uint32_t x_addr = smem_u32(xb) + (lane % 8) * mc.row_stride + (lane / 8) * 16;
+    for (unsigned grp = 0;; ++grp) {
+        const unsigned g = grp % kMmaGroups;
+        if (!warp_wait(&sh.full[g], (grp / kMmaGroups) & 1u, lane, a.status)) return;
+        const Task tk = sh.task[g];
+        if (tk.kind == kTaskEnd) return;
+        const uint32_t w_addr = smem_u32(ring) + (g * kChunk + lane % 8) * mc.row_stride + (lane / 8) * 16;
+        float acc0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, acc1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        for (int ks = ks0; ks < ks0 + per; ks += 2) {
+            uint32_t a0, a2, a0n, a2n, b0, b1, b0n, b1n;
+            ldsm_x4(x_addr + ks * 32, a0, a2, a0n, a2n);
+            ldsm_x4(w_addr + ks * 32, b0, b1, b0n, b1n);
+            mma_bf16_16816(acc0, a0, a2, b0, b1);
+            mma_bf16_16816(acc1, a0n, a2n, b0n, b1n);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sh.empty[g]);
+        // D rows = tokens (lane / 4), columns = rows of the group (2 * (lane % 4) + {0, 1})
+        float* rd = red + ((size_t)g * C + cidx) * 64;
+        const int tok = lane / 4, col = 2 * (lane % 4);
+        rd[tok * 8 + col] = acc0[0] + acc1[0];
+        rd[tok * 8 + col + 1] = acc0[1] + acc1[1];
+        named_bar_sync(1, cthreads);
+        if (cidx < 2) {
+            // add the K slices in warp order: 64 (token, row) values
+            const int i = cidx * 32 + lane;
+            const int t = i / 8, r = i % 8;
+            float v = 0.0f;
+            const float* rg = red + (size_t)g * C * 64;
+#pragma unroll
+            for (int w = 0; w < C; ++w) v += rg[w * 64 + i];
+            volatile ChunkState<NT>& s = sh.cs[tk.cw];
+            const int e = s.e;
+            const int ntok = sh.es.ntok[e];
+            if ((tk.r >> r) & 1) {
+                // token t of the staged activations -> the chunk's batch slot
+#pragma unroll
+                for (int k = 0; k < NT; ++k) {
+                    const int tk_x = a.route ? sh.es.tok[e][k] : k;
+                    if (k < ntok && tk_x == t) {
+                        if (tk.kind == kTaskGate)
+                            s.g[r][k] = v;
+                        else
+                            s.u[r][k] = v;
+                    }
+                }
+            }
+            named_bar_sync(2, 2 * kWarp);
+            if (cidx == 0) {
+                __threadfence_block();
+                if (tk.kind == kTaskGate) {
+                    bool ga = false;
+                    if (lane < kChunk && s.jr[lane] >= 0) {
+#pragma unroll
+                        for (int k = 0; k < NT; ++k) ga |= (k < ntok) && (s.g[lane][k] > 0.0f);
+                    }
+                    const unsigned gm = __ballot_sync(0xffffffffu, ga);
+                    if (lane == 0) s.gmask = gm;
+                    __syncwarp();
+                    __threadfence_block();
+                    if (gm == 0u) finalize_chunk<NT>(a, sh, tk.cw, lane);
+                    if (lane == 0) mbar_arrive(&sh.gate_ready[tk.cw]);
+                } else {
+                    finalize_chunk<NT>(a, sh, tk.cw, lane);
+                }
+            }
+        }
+    }
+}
+
+template <int NT>
+__global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_mma(const FfnLaunch a, const MmaCfg mc) {
+    using T = __nv_bfloat16;
+    constexpr int C = GateUpWarps<NT>::C;
+    __shared__ GateUpShared<NT> sh;
+    extern __shared__ __align__(128) unsigned char dyn[];
+    unsigned char* xb = dyn;                                       // [8][row_stride] bf16 activations
+    float* red = reinterpret_cast<float*>(dyn + (size_t)kChunk * mc.row_stride);  // [2][C][64]
+    unsigned char* ring = dyn + (size_t)kChunk * mc.row_stride + (size_t)kMmaGroups * C * 64 * sizeof(float);
+    const int n_x = a.route ? a.batch : a.nt;
+
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    if (threadIdx.x == 0) {
+        for (int g = 0; g < kMmaGroups; ++g) {
+            mbar_init(&sh.full[g], 1);
+            mbar_init(&sh.empty[g], C);
+        }
+        for (int w = 0; w < kWindow; ++w) {
+            mbar_init(&sh.gate_ready[w], 1);
+            mbar_init(&sh.chunk_free[w], 1);
+        }
+        mbar_fence_init();
+    }
+    const bool early = a.rows == nullptr && a.route == nullptr;
+    if (!early) pdl_wait();
+    resolve_experts(a, sh.es);
+    pdl_launch_dependents();
+
+    const int n_chunks = (a.n_rows + kChunk - 1) / kChunk;
+    const int n_items = sh.es.n_act * n_chunks;
+    const int i0 = (int)((long long)n_items * blockIdx.x / gridDim.x);
+    const int i1 = (int)((long long)n_items * (blockIdx.x + 1) / gridDim.x);
+
+    if (warp == 0) {
+        if (lane == 0) produce_mma<NT>(a, sh, ring, mc, i0, i1, n_chunks);
+        return;
+    }
+    if (early) pdl_wait();
+    const int ctid = threadIdx.x - kWarp;
+    const int cthreads = C * kWarp;
+    const int x_tok0 = a.route ? 0 : a.tok0;
+    // activations as bf16 rows (tokens past the pass are zero)
+    for (int t = 0; t < kChunk; ++t) {
+        __nv_bfloat16* xrow = reinterpret_cast<__nv_bfloat16*>(xb + (size_t)t * mc.row_stride);
+        if (t >= n_x) {
+            for (int i = ctid; i < a.d; i += cthreads) xrow[i] = __float2bfloat16_rn(0.0f);
+        } else if (a.norm_from_h) {
+            const float* hr = a.h + (size_t)(x_tok0 + t) * a.d;
+            float ss = 0.0f;
+            for (int i = ctid; i < a.d; i += cthreads) ss = fmaf(hr[i], hr[i], ss);
+            ss = warp_sum(ss);
+            if (lane == 0) sh.red[warp - 1] = ss;
+            named_bar_sync(1, cthreads);
+            float tot = 0.0f;
+            for (int w = 0; w < C; ++w) tot += sh.red[w];
+            const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)a.d), 1e-5f));
+            for (int i = ctid; i < a.d; i += cthreads)
+                xrow[i] = __float2bfloat16_rn((i == a.d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hr[i], rms)));
+            named_bar_sync(1, cthreads);
+        } else {
+            const T* xr = static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d;
+            for (int i = ctid; i < a.d; i += cthreads) xrow[i] = xr[i];
+        }
+    }
+    named_bar_sync(1, cthreads);
+    consume_mma<NT>(a, sh, ring, xb, red, mc, warp - 1, lane);
+}
+
+static size_t mma_smem(int d, MmaCfg* mc) {
+    mc->row_stride = d * 2 + kMmaRowPad;
+    return (size_t)kChunk * mc->row_stride + (size_t)kMmaGroups * GateUpWarps<8>::C * 64 * sizeof(float) +
+           (size_t)kMmaGroups * kChunk * mc->row_stride;
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 int gate_up_config(int wdtype, int d, int x_tokens, int optin_smem, int* slots, int* slot_bytes,
@@ -707,6 +1000,29 @@ static cudaError_t launch_t(const FfnLaunch& a, int grid, cudaStream_t stream, b
     return cudaLaunchKernelEx(&lc, k_gate_up<T, NT>, a, cfg);
 }
 
+template <int NT>
+static cudaError_t launch_mma_t(const FfnLaunch& a, int grid, cudaStream_t stream, bool pdl) {
+    MmaCfg mc;
+    const size_t smem = mma_smem(a.d, &mc);
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(GateUpWarps<NT>::THREADS);
+    lc.dynamicSmemBytes = smem;
+    lc.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&lc, k_gate_up_mma<NT>, a, mc);
+}
+
+static bool use_mma(int wdtype, int d, int pass_tokens) {
+    MmaCfg mc;
+    return wdtype == 1 && pass_tokens >= 4 && d % kMmaDAlign == 0 &&
+           mma_smem(d, &mc) + kSmemMargin <= (size_t)g_optin;
+}
+
 template <typename T, int NT>
 static cudaError_t prepare_t(int optin) {
     return cudaFuncSetAttribute(k_gate_up<T, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -727,11 +1043,19 @@ cudaError_t prepare_gate_up(int optin_smem) {
     if (e == cudaSuccess) e = prepare_t<float, 2>(optin_smem);
     if (e == cudaSuccess) e = prepare_t<float, 4>(optin_smem);
     if (e == cudaSuccess) e = prepare_t<float, 8>(optin_smem);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_gate_up_mma<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin_smem - kSmemMargin);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_gate_up_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin_smem - kSmemMargin);
     return e;
 }
 
 cudaError_t launch_gate_up(const FfnLaunch& a, int wdtype, int pass_tokens, int grid,
                            cudaStream_t stream, bool pdl) {
+    if (use_mma(wdtype, a.d, pass_tokens)) {
+        if (pass_tokens == 4) return launch_mma_t<4>(a, grid, stream, pdl);
+        if (pass_tokens == 8) return launch_mma_t<8>(a, grid, stream, pdl);
+    }
     if (wdtype == 1) {
         switch (pass_tokens) {
             case 1: return launch_t<__nv_bfloat16, 1>(a, grid, stream, pdl);
