@@ -47,9 +47,9 @@ NOMINAL_HBM_GBS = 7900.0
 # summarised in profiles/k_gate_up-k_down-mistral7b-layer-full.md, and the
 # SHA-256 of the kernel sources it was taken on: once they change, the figure
 # no longer describes the kernel and is reported as null.
-NCU_TRAFFIC = {"bytes": 165.41e6,
+NCU_TRAFFIC = {"bytes": 166.09e6,
                "sources": ("paper_2406_05955_gb300/csrc/ts_gate_up.cu", "paper_2406_05955_gb300/csrc/ts_kernels.cuh"),
-               "sha256": "9d90164aa6d048d3c5feed9a5a7bc4def4982b54a987566d80ed05ee321eb6e5"}
+               "sha256": "50374b962222bce7cc6e72c883b9becb4eb94cdc0a3984ef8e3c4d4be5838de3"}
 
 
 def kernel_sources_sha256(paths) -> str:
@@ -360,7 +360,9 @@ def run_ours(args, dist: Dist) -> dict | None:
     t_gate_up = time_kernel_gate_up(ts, ffns, x, stream, lists, reps=3)
     nb_x = needed_bytes_stack(ffns, lists)  # active sets of the x used in the kernel timing
     peaks = load_peaks()
-    gate_up_bytes = nb_x["gate_up"] / n_layers
+    # passes of 1-2 tokens: the gate+up kernel also gathers the W_down rows
+    # (each CTA's share of the down projection)
+    gate_up_bytes = (nb_x["gate_up"] + (nb_x["down"] if B <= 2 else 0)) / n_layers
     achieved = gate_up_bytes / t_gate_up / 1e9
     step_s = t_max / args.steps
     needed_per_token = (nb["gate_up"] + nb["down"]) / B
@@ -384,7 +386,9 @@ def run_ours(args, dist: Dist) -> dict | None:
             "gate_active_per_layer": statistics.mean(c[0] for c in nb["per_layer_counts"]),
             "both_active_per_layer": statistics.mean(c[1] for c in nb["per_layer_counts"]),
         },
-        "roofline": {"bound": "hbm", "kernel": "k_gate_up (gate GEMV + gathered up projection)",
+        "roofline": {"bound": "hbm",
+                     "kernel": ("k_gate_up (gate GEMV, gathered up projection, this CTA's share of the "
+                                "down projection)" if B <= 2 else "k_gate_up (gate GEMV + gathered up projection)"),
                      "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                      "frac": achieved / peaks["hbm_gbs"], "peak_source": peaks["source"],
                      "traffic": None if predictor or B != 1 else ncu_traffic(),
