@@ -127,8 +127,21 @@ ts_status ts_ffn_get_active(ts_ffn* h, cudaStream_t stream, int token, int32_t* 
                             int* n_gate, int32_t* both_idx, int* n_both);
 
 /* Synchronise `stream`, return and clear the device status word:
-   TS_OK or TS_ERR_BAD_INDEX. */
+   TS_OK, TS_ERR_BAD_INDEX, or TS_ERR_TIMEOUT (a bounded device-side wait ran
+   out; the kernels wound down instead of hanging and the results of that
+   forward are undefined). */
 ts_status ts_ffn_get_error(ts_ffn* h, cudaStream_t stream);
+
+/*
+ * Test hook for the failure-detection path (not part of the method): while
+ * `on` is nonzero, forwards on this handle make one consumer warp of every
+ * gate+up CTA wait on a barrier that nothing arrives at. The wait, like every
+ * device-side wait of the library, gives up after about one second, records
+ * TS_ERR_TIMEOUT in the status word and lets the kernels wind down, so the
+ * CUDA context stays usable. Such a forward takes a few seconds and its
+ * output is undefined. Returns TS_ERR_INVALID_ARG for a NULL handle.
+ */
+ts_status ts_ffn_set_test_stall(ts_ffn* h, int on);
 
 /*
  * One FFN forward with no handle and no device allocation. The paper has no

@@ -41,6 +41,7 @@ SIGNATURES = {
     "ts_stack_forward": (I, [P, I, P, I, P, P, P]),
     "ts_ffn_get_active": (I, [P, P, I, P, IP, P, IP]),
     "ts_ffn_get_error": (I, [P, P]),
+    "ts_ffn_set_test_stall": (I, [P, I]),
     "ts_ffn_forward_noalloc": (I, [I, I, I, P, P, P, P, I, P, P, P, I]),
     "ts_moe_create": (I, [PP, I, I, I, I, P, P, I]),
     "ts_moe_destroy": (None, [P]),
@@ -206,6 +207,10 @@ class Ffn:
 
     def get_error(self, stream=None) -> int:
         return int(lib().ts_ffn_get_error(self.handle, _stream(stream)))
+
+    def set_test_stall(self, on: bool) -> None:
+        """Failure-detection test hook: the next forwards' bounded waits run out."""
+        _check(lib().ts_ffn_set_test_stall(self.handle, int(bool(on))), "ts_ffn_set_test_stall")
 
     def close(self) -> None:
         if getattr(self, "_h", None) is not None:

@@ -100,6 +100,7 @@ struct ts_ffn {
     int last_batch = 0;
     const int32_t* last_rows = nullptr;
     int last_n_rows = 0;
+    int test_stall = 0;  // ts_ffn_set_test_stall
 };
 
 struct ts_moe {
@@ -231,6 +232,7 @@ FfnLaunch ffn_launch(const ts_ffn* h, int batch, const int32_t* rows, int n_rows
     a.status = h->s.status;
     a.partial = h->s.partial;
     a.partial_slots = kAccMaxTokens;
+    a.test_stall = h->test_stall;
     return a;
 }
 
@@ -314,6 +316,7 @@ ts_status read_status(unsigned* status_dev, cudaStream_t stream) {
     if (cudaStreamSynchronize(stream) != cudaSuccess) return TS_ERR_CUDA;
     if (cudaMemcpy(&v, status_dev, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return TS_ERR_CUDA;
     if (cudaMemset(status_dev, 0, sizeof v) != cudaSuccess) return TS_ERR_CUDA;
+    if (v & kStatusTimeout) return TS_ERR_TIMEOUT;
     return (v & kStatusBadIndex) ? TS_ERR_BAD_INDEX : TS_OK;
 }
 
@@ -414,6 +417,12 @@ ts_status ts_ffn_get_active(ts_ffn* h, cudaStream_t stream, int token, int32_t* 
 ts_status ts_ffn_get_error(ts_ffn* h, cudaStream_t stream) {
     if (!h) return TS_ERR_INVALID_ARG;
     return read_status(h->s.status, stream);
+}
+
+ts_status ts_ffn_set_test_stall(ts_ffn* h, int on) {
+    if (!h) return TS_ERR_INVALID_ARG;
+    h->test_stall = on ? 1 : 0;
+    return TS_OK;
 }
 
 // ---------------------------------------------------------------------------

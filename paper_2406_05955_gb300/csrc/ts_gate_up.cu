@@ -88,6 +88,7 @@ struct GateUpShared {
     uint64_t empty[kMaxSlots];
     uint64_t gate_ready[kWindow];
     uint64_t chunk_free[kWindow];
+    uint64_t never;  // nothing arrives here (FfnLaunch::test_stall)
     Task task[kMaxSlots];
     ChunkState<NT> cs[kWindow];
     ExpertSets es;
@@ -308,6 +309,8 @@ __device__ void down_partial(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned 
                     bits = q < kMaxLocal ? (unsigned)sh.pd.ub[q]
                                          : (unsigned)*reinterpret_cast<const volatile uint8_t*>(
                                                a.ubits + (size_t)e * a.nbytes + chunk);
+                    const int left = a.n_rows - chunk * kChunk;  // rows of the row space in this chunk
+                    if (left < kChunk) bits &= (1u << (left > 0 ? left : 0)) - 1u;
                 }
                 const int cnt = __popc(bits);
                 int incl = cnt;
@@ -326,7 +329,8 @@ __device__ void down_partial(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned 
                     for (unsigned b = bits; b; b &= b - 1u) {
                         const int r = __ffs(b) - 1;
                         const int p = chunk * kChunk + r;
-                        const int j = a.rows ? a.rows[p] : p;
+                        int j = a.rows ? a.rows[p] : p;
+                        if ((unsigned)j >= (unsigned)a.m) j = 0;  // only after a failed wait: keep the copy in bounds
                         sh.pd.meta[pos] = make_int2(e, p);
 #pragma unroll
                         for (int t = 0; t < AT; ++t)
@@ -532,6 +536,10 @@ __device__ void consume(const FfnLaunch& a, GateUpShared<NT>& sh, const unsigned
     constexpr int C = GateUpWarps<NT>::C;
     // consumer cidx owns slots cidx, cidx + C, ... (S is a multiple of C)
     unsigned slot = (unsigned)cidx, phase = 0;
+    if (a.test_stall && cidx == 0) {
+        // the failure-detection test: a wait that can only run out
+        if (!warp_wait(&sh.never, 0u, lane, a.status)) return;
+    }
     for (;;) {
         if (!warp_wait(&sh.full[slot], phase, lane, a.status)) return;
         const Task tk = sh.task[slot];
@@ -606,7 +614,11 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up(const F
             mbar_init(&sh.gate_ready[w], 1);
             mbar_init(&sh.chunk_free[w], 1);
         }
-        if constexpr (NT <= kAccMaxTokens) mbar_init(&sh.pd.landed, 1);
+        mbar_init(&sh.never, 1);
+        if constexpr (NT <= kAccMaxTokens) {
+            mbar_init(&sh.pd.landed, 1);
+            for (int q = 0; q < kMaxLocal; ++q) sh.pd.ub[q] = 0;
+        }
         mbar_fence_init();
     }
     // Single FFN in detected mode: nothing the producer reads comes from an

@@ -80,6 +80,10 @@ struct FfnLaunch {
     float* partial;
     int partial_slots;
     int partial_ctas;
+    // Test hook (failure detection): nonzero makes consumer warp 0 of every
+    // gate+up CTA wait on a barrier nothing arrives at, so the bounded wait
+    // runs out and the status word records kStatusTimeout.
+    int test_stall;
     // Stack mode: the next layer's W_gate (nullptr: none), its row count and
     // its gate+up grid. The down-projection CTAs, before waiting for the
     // gate+up kernel, prefetch into L2 the first prefetch_rows rows each
