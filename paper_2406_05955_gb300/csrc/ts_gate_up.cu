@@ -25,7 +25,7 @@
 //     consumers wait before reading the activations.
 //   * Passes of up to kAccMaxTokens tokens also do this CTA's share of the
 //     down projection at the end (down_partial): the CTA's W_down rows are
-//     staged in the idle ring and summed into its block of the partial
+//     read from L2 and summed into its block of the partial
 //     buffer, which the down kernel's reduction adds up over the CTAs.
 // Every mbarrier wait is bounded (kWaitLimitNs); on expiry the status word
 // gets kStatusTimeout and the CTA drains its copies and returns.
@@ -71,13 +71,13 @@ struct ChunkState {
 // needs from each finished chunk (local index q < kMaxLocal; later chunks are
 // read back from global memory), and the staging of its W_down rows.
 constexpr int kMaxLocal = 32;
+constexpr int kRoundCap = 48;  // rows listed per round
 struct PartialShared {
     uint8_t ub[kMaxLocal];                         // both-active rows of chunk q
     float c[kMaxLocal][kChunk][kAccMaxTokens];     // their c values by batch slot
-    int2 meta[kMaxSlots];                          // (expert, position) of the row in each slot
-    float cs[kMaxSlots][kAccMaxTokens];            // its c values
-    int n_rows, next_item;                         // rows staged this round, first item of the next
-    uint64_t landed;                               // every staged row is in its slot
+    const void* rowp[kRoundCap];                   // this round's rows: W_down row address
+    float cs[kRoundCap][kAccMaxTokens];            // and c values
+    int n_rows, next_item;                         // rows listed this round, first item of the next
 };
 struct NoPartial {};
 
@@ -270,42 +270,105 @@ __device__ void finalize_chunk(const FfnLaunch& a, GateUpShared<NT>& sh, int cw,
 // batch slot t,
 //     partial[cta][t][:] = sum over the CTA's both-active rows j, in local
 //                          chunk order and row order, of c_{t,j} W_down[j,:].
-// The ring is idle by then: consumer warp 0 stages up to S rows per round in
-// it by bulk copy (the finalizer already pulled them into L2), then every
-// consumer warp adds its column blocks over the staged rows. A round after
-// the first adds onto the stored partial, so the order stays fixed and the
-// result is bitwise reproducible.
+// Consumer warp 0 lists the rows (their W_down address and c values) in
+// shared memory, kRoundCap per round; every consumer warp then reads its
+// column blocks of those rows straight from L2 (the finalizer prefetched
+// them), all blocks of a group of rows in flight at once, and accumulates in
+// registers. A round after the first adds onto the stored partial, so the
+// order stays fixed and the result is bitwise reproducible.
+template <typename T, int NT, int NB>
+__device__ __forceinline__ void partial_blocks(const FfnLaunch& a, GateUpShared<NT>& sh, int n, int blk0,
+                                               int bstride, float* pbase, bool accumulate, int lane) {
+    constexpr int VEC = Vec<T>::N;
+    constexpr int BLK = kWarp * VEC;
+    constexpr int AT = NT;      // batch slots held (NT <= kAccMaxTokens)
+    constexpr int U = 16 / NB;  // rows per group: 16 loads in flight per lane
+    const int d = a.d;
+    const int n_slots = a.route ? a.batch : a.nt;
+    int col[NB];
+    bool valid[NB];
+    float acc[NB][AT][VEC];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+        col[b] = (blk0 + b * bstride) * BLK + lane * VEC;
+        valid[b] = col[b] < d;
+#pragma unroll
+        for (int t = 0; t < AT; ++t)
+#pragma unroll
+            for (int v = 0; v < VEC; ++v)
+                acc[b][t][v] = (accumulate && valid[b] && t < n_slots) ? pbase[(size_t)t * d + col[b] + v] : 0.0f;
+    }
+    for (int g = 0; g < n; g += U) {
+        uint4 w[U][NB];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const T* row = g + u < n ? reinterpret_cast<const T*>(sh.pd.rowp[g + u]) : nullptr;
+#pragma unroll
+            for (int b = 0; b < NB; ++b)
+                w[u][b] = (row != nullptr && valid[b]) ? ld_stream(row + col[b]) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            if (g + u < n) {
+                float c[AT];
+#pragma unroll
+                for (int t = 0; t < AT; ++t) c[t] = sh.pd.cs[g + u][t];
+#pragma unroll
+                for (int b = 0; b < NB; ++b) {
+                    float f[VEC];
+                    Vec<T>::unpack(w[u][b], f);
+#pragma unroll
+                    for (int t = 0; t < AT; ++t)
+                        if (t < n_slots)
+#pragma unroll
+                            for (int v = 0; v < VEC; ++v) acc[b][t][v] = fmaf(c[t], f[v], acc[b][t][v]);
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int b = 0; b < NB; ++b)
+        if (valid[b]) {
+#pragma unroll
+            for (int t = 0; t < AT; ++t)
+                if (t < n_slots) {
+                    float4* o = reinterpret_cast<float4*>(pbase + (size_t)t * d + col[b]);
+#pragma unroll
+                    for (int v = 0; v < VEC; v += 4)
+                        o[v / 4] = make_float4(acc[b][t][v], acc[b][t][v + 1], acc[b][t][v + 2], acc[b][t][v + 3]);
+                }
+        }
+}
+
 template <typename T, int NT>
-__device__ void down_partial(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char* ring,
-                             const GateUpCfg& cfg, int i0, int i1, int n_chunks, int cidx, int lane) {
+__device__ void down_partial(const FfnLaunch& a, GateUpShared<NT>& sh, int i0, int i1, int n_chunks, int cidx,
+                             int lane) {
     constexpr int VEC = Vec<T>::N;
     constexpr int BLK = kWarp * VEC;
     constexpr int C = GateUpWarps<NT>::C;
     constexpr int AT = kAccMaxTokens;
     const int cthreads = C * kWarp;
     const int d = a.d;
-    const unsigned row_bytes = (unsigned)(d * sizeof(T));
     const int n_slots = a.route ? a.batch : a.nt;
-    const int S = cfg.slots;
     float* pbase = a.partial + (size_t)blockIdx.x * a.partial_slots * d;
     const int nblk = (d + BLK - 1) / BLK;
+    const int my_blocks = cidx < nblk ? (nblk - 1 - cidx) / C + 1 : 0;
     int it = i0;
     unsigned round = 0;
-    bool ok = true;
     do {
         if (cidx == 0) {
-            // stage the rows of the next items, whole items only, at most S rows
+            // the rows of the next items, whole items only, at most kRoundCap
             int n = 0;
             bool full = false;
             while (!full && it < i1) {
                 const int item = it + lane;
+                const int q = item - i0;
                 unsigned bits = 0u;
                 int e = 0, chunk = 0;
                 if (item < i1) {
                     const int ea = item / n_chunks;
                     chunk = item - ea * n_chunks;
                     e = sh.es.act[ea];
-                    const int q = item - i0;
                     bits = q < kMaxLocal ? (unsigned)sh.pd.ub[q]
                                          : (unsigned)*reinterpret_cast<const volatile uint8_t*>(
                                                a.ubits + (size_t)e * a.nbytes + chunk);
@@ -319,91 +382,49 @@ __device__ void down_partial(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned 
                     const int v = __shfl_up_sync(0xffffffffu, incl, o);
                     if (lane >= o) incl += v;
                 }
-                // items that fit this round: a prefix of the lanes
-                const bool fits = item < i1 && n + incl <= S;
+                // the items that fit are a prefix of the lanes
+                const bool fits = item < i1 && n + incl <= kRoundCap;
                 const unsigned take = __ballot_sync(0xffffffffu, fits);
-                const int n_take = __popc(take);  // lanes 0 .. n_take-1
+                const int n_take = __popc(take);
                 if (fits) {
                     int pos = n + incl - cnt;
-                    const int q = item - i0;
                     for (unsigned b = bits; b; b &= b - 1u) {
                         const int r = __ffs(b) - 1;
                         const int p = chunk * kChunk + r;
                         int j = a.rows ? a.rows[p] : p;
-                        if ((unsigned)j >= (unsigned)a.m) j = 0;  // only after a failed wait: keep the copy in bounds
-                        sh.pd.meta[pos] = make_int2(e, p);
+                        if ((unsigned)j >= (unsigned)a.m) j = 0;  // only after a failed wait: stay in bounds
+                        sh.pd.rowp[pos] = static_cast<const T*>(a.ex[e].wd) + (size_t)j * d;
 #pragma unroll
                         for (int t = 0; t < AT; ++t)
                             sh.pd.cs[pos][t] =
                                 q < kMaxLocal ? sh.pd.c[q][r][t]
                                               : (t < n_slots ? a.cval[((size_t)e * kMaxPass + t) * a.cval_tok_stride + p]
                                                              : 0.0f);
-                        mbar_expect_tx(&sh.pd.landed, row_bytes);
-                        tma_load_1d(ring + (size_t)pos * cfg.slot_bytes,
-                                    static_cast<const T*>(a.ex[e].wd) + (size_t)j * d, row_bytes, &sh.pd.landed);
                         ++pos;
                     }
                 }
-                const int added = __shfl_sync(0xffffffffu, incl, n_take > 0 ? n_take - 1 : 0);
-                if (n_take > 0) n += added;
+                if (n_take > 0) n += __shfl_sync(0xffffffffu, incl, n_take - 1);
                 it += n_take;
                 full = n_take < kWarp && it < i1;  // the next item did not fit
             }
-            __syncwarp();
             if (lane == 0) {
                 sh.pd.n_rows = n;
                 sh.pd.next_item = it;
-                mbar_arrive(&sh.pd.landed);  // the phase completes when every copy has landed
             }
         }
         named_bar_sync(1, cthreads);
         const int n = sh.pd.n_rows;
         const int next = sh.pd.next_item;
-        int okw = 1;
-        if (lane == 0) {
-            okw = mbar_wait(&sh.pd.landed, round & 1u) ? 1 : 0;
-            if (!okw) atomicOr(a.status, kStatusTimeout);
-        }
-        if (!__shfl_sync(0xffffffffu, okw, 0)) {
-            // copies still in flight must land before the CTA exits
-            ok = false;
-            if (lane == 0) mbar_wait(&sh.pd.landed, round & 1u);
-            __syncwarp();
-        }
-        if (ok) {
-            for (int blk = cidx; blk < nblk; blk += C) {
-                const int col = blk * BLK + lane * VEC;
-                if (col >= d) continue;
-                float acc[AT][VEC];
-#pragma unroll
-                for (int t = 0; t < AT; ++t)
-#pragma unroll
-                    for (int v = 0; v < VEC; ++v)
-                        acc[t][v] = (round > 0 && t < n_slots) ? pbase[(size_t)t * d + col + v] : 0.0f;
-                for (int i = 0; i < n; ++i) {
-                    float f[VEC];
-                    Vec<T>::unpack(lds128(ring + (size_t)i * cfg.slot_bytes + (size_t)col * sizeof(T)), f);
-#pragma unroll
-                    for (int t = 0; t < AT; ++t) {
-                        const float c = sh.pd.cs[i][t];
-#pragma unroll
-                        for (int v = 0; v < VEC; ++v) acc[t][v] = fmaf(c, f[v], acc[t][v]);
-                    }
-                }
-#pragma unroll
-                for (int t = 0; t < AT; ++t)
-                    if (t < n_slots) {
-                        float4* o = reinterpret_cast<float4*>(pbase + (size_t)t * d + col);
-#pragma unroll
-                        for (int v = 0; v < VEC; v += 4)
-                            o[v / 4] = make_float4(acc[t][v], acc[t][v + 1], acc[t][v + 2], acc[t][v + 3]);
-                    }
-            }
+        if (my_blocks == 2) {
+            partial_blocks<T, NT, 2>(a, sh, n, cidx, C, pbase, round > 0, lane);
+        } else {
+            for (int b = 0; b < my_blocks; ++b)
+                partial_blocks<T, NT, 1>(a, sh, n, cidx + b * C, C, pbase, round > 0, lane);
         }
         it = next;
         ++round;
-        named_bar_sync(1, cthreads);  // the slots and the list are reused next round
-    } while (ok && it < i1);
+        named_bar_sync(1, cthreads);  // the list is rebuilt next round
+    } while (it < i1);
 }
 
 // Single-thread wait that records a timeout in the status word.
@@ -616,7 +637,6 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up(const F
         }
         mbar_init(&sh.never, 1);
         if constexpr (NT <= kAccMaxTokens) {
-            mbar_init(&sh.pd.landed, 1);
             for (int q = 0; q < kMaxLocal; ++q) sh.pd.ub[q] = 0;
         }
         mbar_fence_init();
@@ -668,7 +688,7 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up(const F
         // every chunk is finalized and every ring copy consumed once all
         // consumers are here
         named_bar_sync(1, cthreads);
-        down_partial<T, NT>(a, sh, ring, cfg, i0, i1, n_chunks, warp - 1, lane);
+        down_partial<T, NT>(a, sh, i0, i1, n_chunks, warp - 1, lane);
     }
 }
 
