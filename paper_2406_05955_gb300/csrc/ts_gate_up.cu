@@ -89,6 +89,7 @@ struct GateUpShared {
     uint64_t gate_ready[kWindow];
     uint64_t chunk_free[kWindow];
     uint64_t never;  // nothing arrives here (FfnLaunch::test_stall)
+    int mma_ok;      // tensor-core consumers: every wait so far succeeded
     Task task[kMaxSlots];
     ChunkState<NT> cs[kWindow];
     ExpertSets es;
@@ -841,9 +842,29 @@ __device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsi
     const int per = n_ks / C;           // even: d % kMmaDAlign == 0
     const int ks0 = cidx * per;
     const uint32_t x_addr = smem_u32(xb) + (lane % 8) * mc.row_stride + (lane / 8) * 16;
+    // All consumer warps meet at named barriers inside every group, so they
+    // must agree on whether to go on: one thread waits, the outcome is shared.
+    if (cidx == 0 && lane == 0) {
+        int ok = 1;
+        if (a.test_stall) {
+            // the failure-detection test: a wait that can only run out
+            ok = mbar_wait(&sh.never, 0u) ? 1 : 0;
+            if (!ok) atomicOr(a.status, kStatusTimeout);
+        }
+        sh.mma_ok = ok;
+    }
     for (unsigned grp = 0;; ++grp) {
         const unsigned g = grp % kMmaGroups;
-        if (!warp_wait(&sh.full[g], (grp / kMmaGroups) & 1u, lane, a.status)) return;
+        const unsigned parity = (grp / kMmaGroups) & 1u;
+        if (cidx == 0 && lane == 0 && sh.mma_ok) {
+            const bool ok = mbar_wait(&sh.full[g], parity);
+            if (!ok) atomicOr(a.status, kStatusTimeout);
+            sh.mma_ok = ok ? 1 : 0;
+        }
+        named_bar_sync(1, cthreads);
+        if (!sh.mma_ok) return;
+        // the phase is complete: every thread's own (immediate) wait makes the copies visible to it
+        if (!warp_wait(&sh.full[g], parity, lane, a.status)) return;
         const Task tk = sh.task[g];
         if (tk.kind == kTaskEnd) return;
         const uint32_t w_addr = smem_u32(ring) + (g * kChunk + lane % 8) * mc.row_stride + (lane / 8) * 16;
@@ -928,6 +949,10 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_mma(con
             mbar_init(&sh.full[g], 1);
             mbar_init(&sh.empty[g], C);
         }
+        mbar_init(&sh.never, 1);
+        if constexpr (NT <= kAccMaxTokens) {
+            for (int q = 0; q < kMaxLocal; ++q) sh.pd.ub[q] = 0;
+        }
         for (int w = 0; w < kWindow; ++w) {
             mbar_init(&sh.gate_ready[w], 1);
             mbar_init(&sh.chunk_free[w], 1);
@@ -977,6 +1002,11 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_mma(con
     }
     named_bar_sync(1, cthreads);
     consume_mma<NT>(a, sh, ring, xb, red, mc, warp - 1, lane);
+    if constexpr (NT <= kAccMaxTokens) {
+        // every chunk is finalized once all consumers are here
+        named_bar_sync(1, cthreads);
+        down_partial<T, NT>(a, sh, i0, i1, n_chunks, warp - 1, lane);
+    }
 }
 
 static size_t mma_smem(int d, MmaCfg* mc) {
@@ -1049,9 +1079,11 @@ static cudaError_t launch_mma_t(const FfnLaunch& a, int grid, cudaStream_t strea
     return cudaLaunchKernelEx(&lc, k_gate_up_mma<NT>, a, mc);
 }
 
+constexpr int kMmaMinTokens = 4;  // narrowest bf16 pass that takes the tensor-core variant
+
 static bool use_mma(int wdtype, int d, int pass_tokens) {
     MmaCfg mc;
-    return wdtype == 1 && pass_tokens >= 4 && d % kMmaDAlign == 0 &&
+    return wdtype == 1 && pass_tokens >= kMmaMinTokens && d % kMmaDAlign == 0 &&
            mma_smem(d, &mc) + kSmemMargin <= (size_t)g_optin;
 }
 
@@ -1076,6 +1108,10 @@ cudaError_t prepare_gate_up(int optin_smem) {
     if (e == cudaSuccess) e = prepare_t<float, 4>(optin_smem);
     if (e == cudaSuccess) e = prepare_t<float, 8>(optin_smem);
     if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_gate_up_mma<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin_smem - kSmemMargin);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_gate_up_mma<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin_smem - kSmemMargin);
+    if (e == cudaSuccess)
         e = cudaFuncSetAttribute(k_gate_up_mma<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin_smem - kSmemMargin);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(k_gate_up_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin_smem - kSmemMargin);
@@ -1085,6 +1121,8 @@ cudaError_t prepare_gate_up(int optin_smem) {
 cudaError_t launch_gate_up(const FfnLaunch& a, int wdtype, int pass_tokens, int grid,
                            cudaStream_t stream, bool pdl) {
     if (use_mma(wdtype, a.d, pass_tokens)) {
+        if (pass_tokens == 1) return launch_mma_t<1>(a, grid, stream, pdl);
+        if (pass_tokens == 2) return launch_mma_t<2>(a, grid, stream, pdl);
         if (pass_tokens == 4) return launch_mma_t<4>(a, grid, stream, pdl);
         if (pass_tokens == 8) return launch_mma_t<8>(a, grid, stream, pdl);
     }
