@@ -33,7 +33,8 @@ _LIB = os.path.join(_HERE, "_build", "libtsoracle.so")
 _lock = threading.Lock()
 _lib = None
 
-F32, BF16 = 0, 1
+F32, BF16, INT4 = 0, 1, 2
+INT4_GROUP = 32  # weights per binary16 scale in an INT4 row
 RMS_EPS = 1e-5
 
 
@@ -59,6 +60,8 @@ def _load():
             I = ctypes.c_int
             lib.ts_oracle_ffn.argtypes = [I, I, I, I, P, P, P, P, P, I, P, P, P, P, P, I]
             lib.ts_oracle_ffn.restype = I
+            lib.ts_oracle_ffn_w.argtypes = [I, I, I, I, P, I, P, P, P, P, I, P, P, P, P, P, I]
+            lib.ts_oracle_ffn_w.restype = I
             lib.ts_oracle_router.argtypes = [I, I, I, I, P, P, I, P, P, P]
             lib.ts_oracle_router.restype = I
             lib.ts_oracle_rmsnorm.argtypes = [I, I, P, ctypes.c_double, I, P]
@@ -75,10 +78,11 @@ def max_threads() -> int:
 
 
 def as_array(t) -> np.ndarray:
-    """A torch tensor or numpy array as the oracle's storage: float32 or bf16 bits (uint16)."""
+    """A torch tensor or numpy array as the oracle's storage: float32, bf16 bits
+    (uint16), or INT4 rows (uint8, ``[m][d/2 + d/16]``)."""
     if isinstance(t, np.ndarray):
-        if t.dtype not in (np.float32, np.uint16):
-            raise TypeError(f"oracle arrays are float32 or uint16 (bf16 bits), got {t.dtype}")
+        if t.dtype not in (np.float32, np.uint16, np.uint8):
+            raise TypeError(f"oracle arrays are float32, uint16 (bf16 bits) or uint8 (INT4 rows), got {t.dtype}")
         return np.ascontiguousarray(t)
     import torch  # plain torch CPU ops, only to read a tensor's stored bits
 
@@ -87,11 +91,20 @@ def as_array(t) -> np.ndarray:
         return t.view(torch.int16).numpy().view(np.uint16)
     if t.dtype == torch.float32:
         return t.numpy()
-    raise TypeError(f"oracle tensors are float32 or bfloat16, got {t.dtype}")
+    if t.dtype == torch.uint8:
+        return t.numpy()
+    raise TypeError(f"oracle tensors are float32, bfloat16 or uint8 (INT4 rows), got {t.dtype}")
 
 
 def _dtype_of(a: np.ndarray) -> int:
+    if a.dtype == np.uint8:
+        return INT4
     return BF16 if a.dtype == np.uint16 else F32
+
+
+def int4_row_bytes(d: int) -> int:
+    """Bytes of one INT4 row of d weights: d/2 code bytes and d/32 binary16 scales."""
+    return d // 2 + (d // INT4_GROUP) * 2
 
 
 def _ptr(a: np.ndarray | None):
@@ -101,7 +114,10 @@ def _ptr(a: np.ndarray | None):
 def ffn(x, w_gate, w_up, w_down, rows=None, threads: int = 0) -> dict:
     """Dense dReLU FFN of Eq. 1 + Eq. 2 for a batch of tokens.
 
-    ``x`` is ``[B][d]`` (or ``[d]``), the weights ``[m][d]``, all in one storage type.
+    ``x`` is ``[B][d]`` (or ``[d]``), fp32 or bf16; the weights ``[m][d]`` in the
+    activations' storage type, or all three INT4 rows (uint8 ``[m][d/2 + d/16]``,
+    the weight-only 4-bit storage of the paper's INT4 rows) with bf16 or fp32
+    activations.
     ``rows`` (optional, sorted unique int32) restricts the sum to the listed
     neurons (Sec. 7 predictor mode). Returns float64 ``y [B][d]``, ``g``, ``u``
     ``[B][m]`` and uint8 ``gate_mask`` / ``both_mask`` ``[B][m]``.
@@ -112,8 +128,14 @@ def ffn(x, w_gate, w_up, w_down, rows=None, threads: int = 0) -> dict:
     B, d = x.shape
     m = w_gate.shape[0]
     dt = _dtype_of(x)
+    if dt == INT4:
+        raise ValueError("activations are fp32 or bf16")
+    wdt = _dtype_of(w_gate)
     for w in (w_gate, w_up, w_down):
-        if w.shape != (m, d) or _dtype_of(w) != dt:
+        if wdt == INT4:
+            if d % INT4_GROUP != 0 or w.shape != (m, int4_row_bytes(d)) or _dtype_of(w) != INT4:
+                raise ValueError("INT4 weights must be [m][d/2 + d/16] uint8, d a multiple of 32")
+        elif w.shape != (m, d) or _dtype_of(w) != dt:
             raise ValueError("weights must be [m][d] in the activations' storage type")
     r = None
     n_rows = 0
@@ -125,9 +147,9 @@ def ffn(x, w_gate, w_up, w_down, rows=None, threads: int = 0) -> dict:
     gm = np.zeros((B, m), np.uint8)
     bm = np.zeros((B, m), np.uint8)
     y = np.zeros((B, d), np.float64)
-    rc = _load().ts_oracle_ffn(d, m, B, dt, _ptr(x), _ptr(w_gate), _ptr(w_up), _ptr(w_down),
-                               _ptr(r), n_rows, _ptr(g), _ptr(u), _ptr(gm), _ptr(bm), _ptr(y),
-                               int(threads))
+    rc = _load().ts_oracle_ffn_w(d, m, B, dt, _ptr(x), wdt, _ptr(w_gate), _ptr(w_up), _ptr(w_down),
+                                 _ptr(r), n_rows, _ptr(g), _ptr(u), _ptr(gm), _ptr(bm), _ptr(y),
+                                 int(threads))
     if rc != 0:
         raise ValueError("ts_oracle_ffn rejected its arguments (bad shape or row list)")
     return {"y": y, "g": g, "u": u, "gate_mask": gm, "both_mask": bm}
@@ -220,7 +242,7 @@ def stack(h0, layers, threads: int = 0, record: bool = True) -> dict:
     per_layer = []
     for wg, wu, wd in layers:
         wg = as_array(wg)
-        x = rmsnorm(h, _dtype_of(wg))
+        x = rmsnorm(h, BF16 if _dtype_of(wg) == INT4 else _dtype_of(wg))  # INT4 rows take bf16 activations
         res = ffn(x, wg, wu, wd, threads=threads)
         h_next = (h.astype(np.float64) + res["y"]).astype(np.float32)
         if record:

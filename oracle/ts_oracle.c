@@ -29,7 +29,12 @@
  * with fused multiply-add disabled at build time (-ffp-contract=off), so the
  * result is bit-identical on every host and for every thread count.
  * Inputs are the stored values themselves: fp32, or bf16 bit patterns (the
- * upper 16 bits of an IEEE binary32), decoded exactly to double.
+ * upper 16 bits of an IEEE binary32), decoded exactly to double. Weights may
+ * also be stored as INT4 groups (the weight-only 4-bit storage of the paper's
+ * Mixtral-47B-INT4 rows, Tables 7-9): per neuron row of d weights, d/2 bytes
+ * of 4-bit codes (element i in byte i/2, low nibble for even i) followed by
+ * d/32 IEEE binary16 scales, one per group of 32 consecutive elements; the
+ * weight is scale * (code - 8), decoded exactly to double.
  */
 #include <math.h>
 #include <stdint.h>
@@ -39,7 +44,40 @@
 #include <omp.h>
 #endif
 
-enum { ORACLE_F32 = 0, ORACLE_BF16 = 1 };
+enum { ORACLE_F32 = 0, ORACLE_BF16 = 1, ORACLE_INT4 = 2 };
+
+/* Exact IEEE binary16 -> double (by the bit definition). */
+static double half_to_double(uint16_t h) {
+    const int sgn = h >> 15, e = (h >> 10) & 31, f = h & 1023;
+    double v;
+    if (e == 0)
+        v = ldexp((double)f, -24); /* subnormal: f * 2^-24 */
+    else if (e == 31)
+        v = f ? NAN : INFINITY;
+    else
+        v = ldexp((double)(f + 1024), e - 25); /* (1 + f/1024) * 2^(e-15) */
+    return sgn ? -v : v;
+}
+
+/* Bytes of one INT4 row of d weights. */
+static size_t int4_row_bytes(int d) { return (size_t)d / 2 + (size_t)(d / 32) * 2; }
+
+/* Weight (j, i) of a [m][d] matrix stored as wdtype. */
+static double welem(const void* base, int wdtype, int d, int j, int i) {
+    if (wdtype != ORACLE_INT4) {
+        const size_t idx = (size_t)j * (size_t)d + (size_t)i;
+        if (wdtype == ORACLE_F32) return (double)((const float*)base)[idx];
+        uint32_t bits = (uint32_t)((const uint16_t*)base)[idx] << 16;
+        float f;
+        memcpy(&f, &bits, sizeof f);
+        return (double)f;
+    }
+    const uint8_t* row = (const uint8_t*)base + (size_t)j * int4_row_bytes(d);
+    const int code = (row[i / 2] >> (4 * (i & 1))) & 15;
+    const uint8_t* sp = row + d / 2 + (size_t)(i / 32) * 2;
+    const uint16_t h = (uint16_t)(sp[0] | (sp[1] << 8)); /* little-endian */
+    return half_to_double(h) * (double)(code - 8);
+}
 
 /* Exact decode of one stored element to double. */
 static double elem(const void* base, int dtype, size_t idx) {
@@ -72,8 +110,9 @@ int ts_oracle_max_threads(void) {
 /*
  * Dense definition of the dReLU Gated-MLP (Eq. 1 with Eq. 2) for B tokens.
  *
- *   x        [B][d]  activations (dtype)
- *   w_gate   [m][d]  w_up [m][d]  w_down [m][d]  (dtype)
+ *   x        [B][d]  activations (dtype: fp32 or bf16)
+ *   w_gate   [m][d]  w_up [m][d]  w_down [m][d]  (wdtype: fp32, bf16, or
+ *            INT4 rows of d/2 code bytes + d/32 binary16 scales)
  *   rows     NULL: every neuron 0..m-1 takes part.
  *            else: the n_rows listed neurons only (Sec. 7 predictor mode);
  *            the list must be strictly ascending and inside [0, m).
@@ -86,11 +125,13 @@ int ts_oracle_max_threads(void) {
  *
  * Returns 0, or -1 if an argument is invalid (nothing is written then).
  */
-int ts_oracle_ffn(int d, int m, int B, int dtype, const void* x, const void* w_gate,
-                  const void* w_up, const void* w_down, const int32_t* rows, int n_rows,
-                  double* g, double* u, uint8_t* gate_mask, uint8_t* both_mask, double* y,
-                  int n_threads) {
+int ts_oracle_ffn_w(int d, int m, int B, int dtype, const void* x, int wdtype, const void* w_gate,
+                    const void* w_up, const void* w_down, const int32_t* rows, int n_rows,
+                    double* g, double* u, uint8_t* gate_mask, uint8_t* both_mask, double* y,
+                    int n_threads) {
     if (d <= 0 || m <= 0 || B < 0 || (dtype != ORACLE_F32 && dtype != ORACLE_BF16)) return -1;
+    if (wdtype != ORACLE_F32 && wdtype != ORACLE_BF16 && wdtype != ORACLE_INT4) return -1;
+    if (wdtype == ORACLE_INT4 && d % 32 != 0) return -1;
     if (rows != NULL) {
         if (n_rows < 0 || n_rows > m) return -1;
         for (int p = 0; p < n_rows; ++p) {
@@ -125,11 +166,10 @@ int ts_oracle_ffn(int d, int m, int B, int dtype, const void* x, const void* w_g
         for (int j = 0; j < m; ++j) {
             double gj = 0.0, uj = 0.0;
             if (part[j]) {
-                const size_t wo = (size_t)j * (size_t)d;
                 for (int i = 0; i < d; ++i) {
                     double xi = elem(x, dtype, xo + (size_t)i);
-                    gj += elem(w_gate, dtype, wo + (size_t)i) * xi;
-                    uj += elem(w_up, dtype, wo + (size_t)i) * xi;
+                    gj += welem(w_gate, wdtype, d, j, i) * xi;
+                    uj += welem(w_up, wdtype, d, j, i) * xi;
                 }
             }
             gb[j] = gj;
@@ -149,12 +189,21 @@ int ts_oracle_ffn(int d, int m, int B, int dtype, const void* x, const void* w_g
             if (!part[j]) continue;
 #pragma omp for schedule(static)
             for (int i = 0; i < d; ++i)
-                yb[i] += c[j] * elem(w_down, dtype, (size_t)j * (size_t)d + (size_t)i);
+                yb[i] += c[j] * welem(w_down, wdtype, d, j, i);
         }
     }
     free(part);
     free(c);
     return 0;
+}
+
+/* As ts_oracle_ffn_w with weights stored like the activations. */
+int ts_oracle_ffn(int d, int m, int B, int dtype, const void* x, const void* w_gate,
+                  const void* w_up, const void* w_down, const int32_t* rows, int n_rows,
+                  double* g, double* u, uint8_t* gate_mask, uint8_t* both_mask, double* y,
+                  int n_threads) {
+    return ts_oracle_ffn_w(d, m, B, dtype, x, dtype, w_gate, w_up, w_down, rows, n_rows, g, u,
+                           gate_mask, both_mask, y, n_threads);
 }
 
 /*

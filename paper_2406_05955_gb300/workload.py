@@ -82,6 +82,62 @@ def ffn_layer(d: int, m: int, *, activation: float = 0.10, mu: float | None = No
                     wd.to(dtype).contiguous(), b.float())
 
 
+# ---------------------------------------------------------------------------
+# INT4 weight storage (the weight-only 4-bit rows of the paper's INT4 models,
+# Tables 7-9): per neuron row of d weights, d/2 bytes of 4-bit codes (element
+# i in byte i/2, low nibble for even i) followed by d/32 IEEE binary16 scales
+# (little-endian), one per group of 32 consecutive elements. A stored weight
+# is scale * (code - 8).
+# ---------------------------------------------------------------------------
+INT4_GROUP = 32
+
+
+def int4_row_bytes(d: int) -> int:
+    return d // 2 + (d // INT4_GROUP) * 2
+
+
+def quantize_int4(w: torch.Tensor) -> torch.Tensor:
+    """Round ``[m][d]`` weights to INT4 rows (uint8 ``[m][d/2 + d/16]``).
+
+    Per group of 32: scale = max|w| / 7 rounded to binary16 (1 where the group
+    is all zero), code = clamp(round(w / scale), -8, 7) + 8.
+    """
+    m, d = w.shape
+    if d % INT4_GROUP:
+        raise ValueError("d must be a multiple of 32 for INT4 rows")
+    wf = w.detach().float().reshape(m, d // INT4_GROUP, INT4_GROUP)
+    scale = (wf.abs().amax(-1) / 7.0).to(torch.float16)
+    scale = torch.where(scale == 0, torch.ones_like(scale), scale)
+    q = torch.clamp(torch.round(wf / scale.float().unsqueeze(-1)), -8, 7).to(torch.int32) + 8
+    q = q.reshape(m, d)
+    codes = (q[:, 0::2] | (q[:, 1::2] << 4)).to(torch.uint8)
+    scales = scale.contiguous().view(torch.uint8).reshape(m, (d // INT4_GROUP) * 2)
+    return torch.cat([codes, scales], dim=1).contiguous()
+
+
+@dataclass
+class FfnLayerInt4:
+    """One dReLU FFN's INT4 rows (uint8 ``[m][d/2 + d/16]`` each) and the offsets they were drawn with."""
+    w_gate: torch.Tensor
+    w_up: torch.Tensor
+    w_down: torch.Tensor
+    offsets: torch.Tensor
+    d: int
+
+    @property
+    def m(self) -> int:
+        return int(self.w_gate.shape[0])
+
+
+def ffn_layer_int4(d: int, m: int, *, activation: float = 0.10, mu: float | None = None,
+                   sigma_b: float = SIGMA_B, seed: int = 0, device="cpu") -> FfnLayerInt4:
+    """Draw a layer as ``ffn_layer`` does (fp32), then store it as INT4 rows."""
+    L = ffn_layer(d, m, activation=activation, mu=mu, sigma_b=sigma_b, dtype=torch.float32, seed=seed,
+                  device=device)
+    return FfnLayerInt4(quantize_int4(L.w_gate), quantize_int4(L.w_up), quantize_int4(L.w_down),
+                        L.offsets, d)
+
+
 def tokens(B: int, d: int, *, dtype=torch.bfloat16, seed: int = 0, device="cpu") -> torch.Tensor:
     """Token activations ``[B][d]``: N(0,1) entries with the bias channel ``x[:, d-1] = 1``."""
     x = torch.randn(B, d, generator=_gen(seed, device), device=device)
