@@ -49,7 +49,16 @@ typedef enum {
     TS_ERR_UNSUPPORTED = 6   /* valid request this build does not handle     */
 } ts_status;
 
-typedef enum { TS_F32 = 0, TS_BF16 = 1 } ts_dtype;
+/*
+ * Weight storage. TS_F32 and TS_BF16 rows hold d elements. TS_INT4 rows (the
+ * weight-only 4-bit storage of the paper's INT4 models, Tables 7-9) hold d/2
+ * bytes of 4-bit codes -- element i in byte i/2, the low nibble for even i --
+ * followed by d/32 little-endian IEEE binary16 scales, one per group of 32
+ * consecutive elements: weight i = scale[i/32] * (code[i] - 8). An INT4 row
+ * is 9d/16 bytes and needs d to be a multiple of 256; its activations x are
+ * bf16.
+ */
+typedef enum { TS_F32 = 0, TS_BF16 = 1, TS_INT4 = 2 } ts_dtype;
 
 typedef struct ts_ffn ts_ffn;     /* one dReLU FFN (one layer or one expert) */
 typedef struct ts_moe ts_moe;     /* one top-k MoE layer over ts_ffn experts */
@@ -64,9 +73,11 @@ int ts_version(void);
 /*
  * Create a handle for one dReLU FFN (Eq. 1 + Eq. 2).
  *   d, m       model width and number of neurons (d >= 1, m >= 1)
- *   wdtype     storage type of weights and activations
- *   w_gate, w_up, w_down  device pointers, [m][d] each (borrowed)
- *   max_batch  largest batch a forward may pass (1..64)
+ *   wdtype     storage type of the weights (and of x, except INT4: bf16 x)
+ *   w_gate, w_up, w_down  device pointers, [m][d] each, or [m][9d/16] bytes
+ *              for TS_INT4 (borrowed)
+ *   max_batch  largest batch a forward may pass (1..64); INT4 handles run
+ *              passes of up to 2 tokens
  * Allocates the handle's scratch on the current device.
  * Returns TS_ERR_INVALID_ARG for bad sizes/pointers/alignment, TS_ERR_OOM if
  * scratch cannot be allocated, TS_ERR_CUDA for other CUDA failures.
@@ -178,9 +189,11 @@ ts_status ts_ffn_forward_noalloc(int d, int m, ts_dtype wdtype, const void* w_ga
  *     tie), w = softmax over the picked logits,
  *     y_t = sum_k w_{t,k} * FFN_{e_{t,k}}(x_t),
  * each expert itself a neuron-sparse dReLU FFN.
- *   w_router   device [n_experts][d], wdtype (borrowed)
+ *   w_router   device [n_experts][d], wdtype (bf16 when the experts are
+ *              TS_INT4; borrowed)
  *   experts    n_experts handles (same d and wdtype; borrowed)
- *   n_experts  1..16, top_k 1..min(4, n_experts), max_batch 1..8
+ *   n_experts  1..16, top_k 1..min(4, n_experts), max_batch 1..8 (1..2 for
+ *              INT4 experts)
  */
 ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype wdtype,
                         const void* w_router, ts_ffn* const* experts, int max_batch);

@@ -19,7 +19,7 @@ LIB_PATH = os.path.join(_HERE, "_build", "libtsffn.so")
 
 TS_OK, TS_ERR_INVALID_ARG, TS_ERR_CUDA, TS_ERR_OOM, TS_ERR_BAD_INDEX, TS_ERR_TIMEOUT, \
     TS_ERR_UNSUPPORTED = range(7)
-TS_F32, TS_BF16 = 0, 1
+TS_F32, TS_BF16, TS_INT4 = 0, 1, 2
 
 _lock = threading.Lock()
 _lib = None
@@ -137,22 +137,30 @@ def _list(active_idx):
 
 
 class Ffn:
-    """One dReLU FFN layer (or MoE expert) over borrowed ``[m][d]`` device weights."""
+    """One dReLU FFN layer (or MoE expert) over borrowed device weights: ``[m][d]``
+    bf16 / fp32, or INT4 rows (uint8 ``[m][9d/16]``, with bf16 activations)."""
 
     def __init__(self, w_gate: torch.Tensor, w_up: torch.Tensor, w_down: torch.Tensor,
                  max_batch: int = 1):
         for t, n in ((w_gate, "w_gate"), (w_up, "w_up"), (w_down, "w_down")):
             _dev(t, n)
-        m, d = w_gate.shape
-        if w_up.shape != (m, d) or w_down.shape != (m, d):
-            raise ValueError("w_gate, w_up, w_down must all be [m][d]")
         if not (w_gate.dtype == w_up.dtype == w_down.dtype):
             raise TypeError("weights must share one dtype")
+        m, cols = w_gate.shape
+        if w_gate.dtype == torch.uint8:
+            d = cols * 16 // 9
+            if d % 256 or d // 2 + d // 16 != cols:
+                raise ValueError("INT4 rows must be [m][9d/16] bytes with d a multiple of 256")
+            self.wcode, self.dtype = TS_INT4, torch.bfloat16
+        else:
+            d = cols
+            self.wcode, self.dtype = _dtype_code(w_gate), w_gate.dtype
+        if w_up.shape != (m, cols) or w_down.shape != (m, cols):
+            raise ValueError("w_gate, w_up, w_down must have one shape")
         self.d, self.m, self.max_batch = int(d), int(m), int(max_batch)
-        self.dtype = w_gate.dtype
         self._keep = (w_gate, w_up, w_down)
         h = ctypes.c_void_p()
-        _check(lib().ts_ffn_create(ctypes.byref(h), self.d, self.m, _dtype_code(w_gate),
+        _check(lib().ts_ffn_create(ctypes.byref(h), self.d, self.m, self.wcode,
                                    w_gate.data_ptr(), w_up.data_ptr(), w_down.data_ptr(),
                                    self.max_batch), "ts_ffn_create")
         self._h = h
@@ -294,7 +302,7 @@ class Moe:
         self._keep = (w_router,)
         arr = _handles(self.experts)
         h = ctypes.c_void_p()
-        _check(lib().ts_moe_create(ctypes.byref(h), self.d, self.E, self.top_k, _dtype_code(w_router),
+        _check(lib().ts_moe_create(ctypes.byref(h), self.d, self.E, self.top_k, self.experts[0].wcode,
                                    w_router.data_ptr(), _addr(arr), self.max_batch), "ts_moe_create")
         self._h = h
         self.m = self.experts[0].m

@@ -21,7 +21,13 @@ constexpr int kPrefetchRows = 32;
 
 size_t align_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
-int elem_size(ts_dtype dt) { return dt == TS_BF16 ? 2 : 4; }
+int elem_size(ts_dtype dt) { return dt == TS_BF16 ? 2 : 4; }  // fp32 / bf16 weights
+// activations: bf16 for bf16 and INT4 weights, fp32 for fp32 weights
+int act_size(ts_dtype dt) { return dt == TS_F32 ? 4 : 2; }
+ts_dtype act_dtype(ts_dtype dt) { return dt == TS_F32 ? TS_F32 : TS_BF16; }
+size_t weight_row_bytes(ts_dtype dt, int d) {
+    return dt == TS_INT4 ? (size_t)d / 2 + (size_t)(d / 32) * 2 : (size_t)d * elem_size(dt);
+}
 int pow2_tokens(int nt) { return nt <= 1 ? 1 : nt <= 2 ? 2 : nt <= 4 ? 4 : 8; }
 
 // Device facts needed to size grids; looked up at handle creation.
@@ -101,6 +107,7 @@ struct ts_ffn {
     const int32_t* last_rows = nullptr;
     int last_n_rows = 0;
     int test_stall = 0;  // ts_ffn_set_test_stall
+    int pass_max = kMaxPass;  // tokens per pass (kAccMaxTokens for INT4 rows)
 };
 
 struct ts_moe {
@@ -145,17 +152,20 @@ ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void*
     if (out == nullptr) return TS_ERR_INVALID_ARG;
     *out = nullptr;
     if (d < 1 || m < 1 || max_batch < 1 || max_batch > kMaxBatch) return TS_ERR_INVALID_ARG;
-    if (wdtype != TS_F32 && wdtype != TS_BF16) return TS_ERR_INVALID_ARG;
+    if (wdtype != TS_F32 && wdtype != TS_BF16 && wdtype != TS_INT4) return TS_ERR_INVALID_ARG;
     if (!w_gate || !w_up || !w_down) return TS_ERR_INVALID_ARG;
     if (!aligned16(w_gate) || !aligned16(w_up) || !aligned16(w_down)) return TS_ERR_INVALID_ARG;
-    if (((size_t)d * elem_size(wdtype)) % 16 != 0) return TS_ERR_INVALID_ARG;
+    if (wdtype == TS_INT4 ? d % 256 != 0 : ((size_t)d * elem_size(wdtype)) % 16 != 0) return TS_ERR_INVALID_ARG;
     if (m > (1 << 28) || (size_t)d * (size_t)m > ((size_t)1 << 40)) return TS_ERR_UNSUPPORTED;
 
     DeviceInfo dev;
     ts_status st = device_info(&dev);
     if (st != TS_OK) return st;
-    const int pass_cap = std::min(max_batch, kMaxPass);
-    {
+    const int pass_max = wdtype == TS_INT4 ? kAccMaxTokens : kMaxPass;  // INT4: passes of 1-2 tokens
+    const int pass_cap = std::min(max_batch, pass_max);
+    if (wdtype == TS_INT4) {
+        if (!int4_supported(d, pass_cap, dev.optin_smem)) return TS_ERR_UNSUPPORTED;
+    } else {
         int slots, slot_bytes, xs_stride;
         size_t smem;
         if (gate_up_config(wdtype, d, pass_cap, dev.optin_smem, &slots, &slot_bytes, &xs_stride, &smem) != 0)
@@ -172,6 +182,7 @@ ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void*
     h->wu = w_up;
     h->wd = w_down;
     h->dev = dev;
+    h->pass_max = pass_max;
     h->nbytes = (m + 31) / 32 * 4;
     const int n_chunks = (m + kChunk - 1) / kChunk;
     for (int nt : {1, 2, 4, 8}) h->grid[nt] = std::max(1, std::min(dev.num_sms, n_chunks));
@@ -213,7 +224,8 @@ FfnLaunch ffn_launch(const ts_ffn* h, int batch, const int32_t* rows, int n_rows
     memset(&a, 0, sizeof a);
     a.d = h->d;
     a.m = h->m;
-    a.elem_bytes = elem_size(h->dt);
+    a.elem_bytes = h->dt == TS_INT4 ? 0 : elem_size(h->dt);
+    a.row_bytes = (int)weight_row_bytes(h->dt, h->d);
     a.rows = rows;
     a.n_rows = rows ? n_rows : h->m;
     a.batch = batch;
@@ -334,8 +346,8 @@ ts_status ts_ffn_forward(ts_ffn* h, const void* x, int batch, float* y, cudaStre
     FfnLaunch a = ffn_launch(h, batch, active_idx, n_active);
     a.x = x;
     a.y = y;
-    for (int t0 = 0; t0 < batch; t0 += kMaxPass) {
-        st = run_pass(h, a, t0, std::min(kMaxPass, batch - t0), stream, true, true);
+    for (int t0 = 0; t0 < batch; t0 += h->pass_max) {
+        st = run_pass(h, a, t0, std::min(h->pass_max, batch - t0), stream, true, true);
         if (st != TS_OK) return st;
     }
     remember(h, batch, active_idx, n_active);
@@ -345,7 +357,7 @@ ts_status ts_ffn_forward(ts_ffn* h, const void* x, int batch, float* y, cudaStre
 ts_status ts_ffn_gate_up(ts_ffn* h, const void* x, int batch, cudaStream_t stream,
                          const int32_t* active_idx, int n_active) {
     if (!h || batch < 0 || batch > h->max_batch) return TS_ERR_INVALID_ARG;
-    if (batch > kMaxPass) return TS_ERR_UNSUPPORTED;
+    if (batch > h->pass_max) return TS_ERR_UNSUPPORTED;
     if (batch == 0) return TS_OK;
     if (!x) return TS_ERR_INVALID_ARG;
     ts_status st = check_list(h, active_idx, n_active);
@@ -358,7 +370,7 @@ ts_status ts_ffn_gate_up(ts_ffn* h, const void* x, int batch, cudaStream_t strea
 }
 
 ts_status ts_ffn_down(ts_ffn* h, int batch, float* y, cudaStream_t stream) {
-    if (!h || batch < 0 || batch > kMaxPass) return TS_ERR_INVALID_ARG;
+    if (!h || batch < 0 || batch > h->pass_max) return TS_ERR_INVALID_ARG;
     if (batch == 0) return TS_OK;
     if (!y || batch != h->last_batch) return TS_ERR_INVALID_ARG;
     FfnLaunch a = ffn_launch(h, batch, h->last_rows, h->last_n_rows);
@@ -389,14 +401,14 @@ ts_status ts_stack_forward(ts_ffn* const* layers, int n_layers, float* hres, int
         a.norm_from_h = 1;
         a.residual_out = 1;
         const bool next_dense = l + 1 < n_layers && !(active_idx && active_idx[l + 1]);
-        if (next_dense && batch <= kMaxPass) {
+        if (next_dense && batch <= kMaxPass && h->dt != TS_INT4) {
             a.next_wg = layers[l + 1]->wg;
             a.next_n_rows = layers[l + 1]->m;
             a.next_grid = layers[l + 1]->grid[pow2_tokens(std::min(kMaxPass, batch))];
             a.prefetch_rows = kPrefetchRows;
         }
-        for (int t0 = 0; t0 < batch; t0 += kMaxPass) {
-            ts_status st = run_pass(h, a, t0, std::min(kMaxPass, batch - t0), stream, true, true);
+        for (int t0 = 0; t0 < batch; t0 += h->pass_max) {
+            ts_status st = run_pass(h, a, t0, std::min(h->pass_max, batch - t0), stream, true, true);
             if (st != TS_OK) return st;
         }
         remember(h, batch, rows, nr);
@@ -435,8 +447,9 @@ ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype 
     if (d < 1 || n_experts < 1 || n_experts > kMaxExperts) return TS_ERR_INVALID_ARG;
     if (top_k < 1 || top_k > std::min(kMaxTopK, n_experts)) return TS_ERR_INVALID_ARG;
     if (max_batch < 1 || max_batch > kMaxMoeBatch) return TS_ERR_INVALID_ARG;
-    if (wdtype != TS_F32 && wdtype != TS_BF16) return TS_ERR_INVALID_ARG;
+    if (wdtype != TS_F32 && wdtype != TS_BF16 && wdtype != TS_INT4) return TS_ERR_INVALID_ARG;
     if (!w_router || !aligned16(w_router) || !experts) return TS_ERR_INVALID_ARG;
+    if (wdtype == TS_INT4 && max_batch > kAccMaxTokens) return TS_ERR_UNSUPPORTED;
     if (d > kRouterMaxD) return TS_ERR_UNSUPPORTED;
     for (int e = 0; e < n_experts; ++e) {
         const ts_ffn* x = experts[e];
@@ -445,7 +458,9 @@ ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype 
     DeviceInfo dev;
     ts_status st = device_info(&dev);
     if (st != TS_OK) return st;
-    {
+    if (wdtype == TS_INT4) {
+        if (!int4_supported(d, max_batch, dev.optin_smem)) return TS_ERR_UNSUPPORTED;
+    } else {
         int slots, slot_bytes, xs_stride;
         size_t smem;
         if (gate_up_config(wdtype, d, max_batch, dev.optin_smem, &slots, &slot_bytes, &xs_stride, &smem) != 0)
@@ -476,7 +491,7 @@ ts_status ts_moe_create(ts_moe** out, int d, int n_experts, int top_k, ts_dtype 
     const size_t o_ug = h->arena.take((size_t)E * h->nbytes);
     const size_t o_s = h->arena.take(sizeof(unsigned));
     const size_t o_r = h->arena.take((size_t)max_batch * sizeof(TokenRoute));
-    const size_t o_x = h->arena.take((size_t)max_batch * d * elem_size(wdtype));
+    const size_t o_x = h->arena.take((size_t)max_batch * d * act_size(wdtype));
     st = alloc_arena(&h->arena);
     if (st != TS_OK) {
         delete h;
@@ -518,14 +533,16 @@ ts_status moe_layer(ts_moe* h, const void* x, float* hres, int batch, float* y, 
     r.xbuf = h->xbuf;
     r.wr = h->wr;
     r.route = h->route;
-    ts_status st = cuda_status(launch_router(r, h->dt, stream, true));
+    // the router and its normalised activations use the activation type
+    ts_status st = cuda_status(launch_router(r, act_dtype(h->dt), stream, true));
     if (st != TS_OK) return st;
 
     FfnLaunch a;
     memset(&a, 0, sizeof a);
     a.d = h->d;
     a.m = h->m;
-    a.elem_bytes = elem_size(h->dt);
+    a.elem_bytes = h->dt == TS_INT4 ? 0 : elem_size(h->dt);
+    a.row_bytes = (int)weight_row_bytes(h->dt, h->d);
     a.n_rows = h->m;
     a.rows = nullptr;
     a.batch = batch;

@@ -220,8 +220,8 @@ __device__ void finalize_chunk(const FfnLaunch& a, GateUpShared<NT>& sh, int cw,
     // The down projection will gather these W_down rows: pull them into L2
     // now, while HBM is streaming anyway.
     if (lane < kChunk && ((ub >> lane) & 1u))
-        prefetch_l2_bulk(static_cast<const unsigned char*>(a.ex[e].wd) + (size_t)j * a.d * a.elem_bytes,
-                         (unsigned)(a.d * a.elem_bytes));
+        prefetch_l2_bulk(static_cast<const unsigned char*>(a.ex[e].wd) + (size_t)j * a.row_bytes,
+                         (unsigned)a.row_bytes);
     // c by batch slot: the pass-local token (single FFN) or the global token
     // (MoE, 0 for tokens not routed to this expert)
     if (lane < kChunk && ((ub >> lane) & 1u)) {
@@ -341,7 +341,76 @@ __device__ __forceinline__ void partial_blocks(const FfnLaunch& a, GateUpShared<
         }
 }
 
-template <typename T, int NT>
+// INT4 rows: lane l of a warp covers 16 columns (8 code bytes, half a group,
+// one scale) of a 512-column block, for U rows at a time.
+__device__ __forceinline__ uint2 ld_nc_u2(const void* p) {
+    uint2 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(p));
+    return v;
+}
+__device__ __forceinline__ float ld_nc_half(const void* p) {
+    unsigned short v;
+    asm volatile("ld.global.nc.u16 %0, [%1];" : "=h"(v) : "l"(p));
+    return __half2float(__ushort_as_half(v));
+}
+
+template <int NT>
+__device__ __forceinline__ void partial_blocks_q4(const FfnLaunch& a, GateUpShared<NT>& sh, int n, int blk,
+                                                  float* pbase, bool accumulate, int lane) {
+    constexpr int AT = NT;
+    constexpr int U = 8;
+    const int d = a.d;
+    const int n_slots = a.route ? a.batch : a.nt;
+    const int col = blk * 512 + lane * 16;
+    const bool valid = col < d;
+    float acc[AT][16];
+#pragma unroll
+    for (int t = 0; t < AT; ++t)
+#pragma unroll
+        for (int v = 0; v < 16; ++v)
+            acc[t][v] = (accumulate && valid && t < n_slots) ? pbase[(size_t)t * d + col + v] : 0.0f;
+    for (int g = 0; g < n; g += U) {
+        uint2 cw[U];
+        float sc[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const unsigned char* row = g + u < n ? static_cast<const unsigned char*>(sh.pd.rowp[g + u]) : nullptr;
+            cw[u] = make_uint2(0x88888888u, 0x88888888u);  // codes of weight 0
+            sc[u] = 0.0f;
+            if (row != nullptr && valid) {
+                cw[u] = ld_nc_u2(row + col / 2);
+                sc[u] = ld_nc_half(row + d / 2 + (col / 32) * 2);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            if (g + u < n) {
+                float c[AT];
+#pragma unroll
+                for (int t = 0; t < AT; ++t) c[t] = sh.pd.cs[g + u][t] * sc[u];
+#pragma unroll
+                for (int v = 0; v < 16; ++v) {
+                    const uint32_t word = v < 8 ? cw[u].x : cw[u].y;
+                    const float q = (float)((int)((word >> (4 * (v & 7))) & 15u) - 8);
+#pragma unroll
+                    for (int t = 0; t < AT; ++t)
+                        if (t < n_slots) acc[t][v] = fmaf(c[t], q, acc[t][v]);
+                }
+            }
+        }
+    }
+    if (valid) {
+#pragma unroll
+        for (int t = 0; t < AT; ++t)
+            if (t < n_slots) {
+                float4* o = reinterpret_cast<float4*>(pbase + (size_t)t * d + col);
+#pragma unroll
+                for (int v = 0; v < 16; v += 4) o[v / 4] = make_float4(acc[t][v], acc[t][v + 1], acc[t][v + 2], acc[t][v + 3]);
+            }
+    }
+}
+
+template <typename T, int NT, bool Q4 = false>
 __device__ void down_partial(const FfnLaunch& a, GateUpShared<NT>& sh, int i0, int i1, int n_chunks, int cidx,
                              int lane) {
     constexpr int VEC = Vec<T>::N;
@@ -394,7 +463,7 @@ __device__ void down_partial(const FfnLaunch& a, GateUpShared<NT>& sh, int i0, i
                         const int p = chunk * kChunk + r;
                         int j = a.rows ? a.rows[p] : p;
                         if ((unsigned)j >= (unsigned)a.m) j = 0;  // only after a failed wait: stay in bounds
-                        sh.pd.rowp[pos] = static_cast<const T*>(a.ex[e].wd) + (size_t)j * d;
+                        sh.pd.rowp[pos] = static_cast<const unsigned char*>(a.ex[e].wd) + (size_t)j * a.row_bytes;
 #pragma unroll
                         for (int t = 0; t < AT; ++t)
                             sh.pd.cs[pos][t] =
@@ -416,7 +485,9 @@ __device__ void down_partial(const FfnLaunch& a, GateUpShared<NT>& sh, int i0, i
         named_bar_sync(1, cthreads);
         const int n = sh.pd.n_rows;
         const int next = sh.pd.next_item;
-        if (my_blocks == 2) {
+        if constexpr (Q4) {
+            for (int b = cidx; b < (d + 511) / 512; b += C) partial_blocks_q4<NT>(a, sh, n, b, pbase, round > 0, lane);
+        } else if (my_blocks == 2) {
             partial_blocks<T, NT, 2>(a, sh, n, cidx, C, pbase, round > 0, lane);
         } else {
             for (int b = 0; b < my_blocks; ++b)
@@ -726,21 +797,24 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint3
 }
 
 struct MmaCfg {
-    int row_stride;  // bytes per row in shared memory (d * 2 + kMmaRowPad)
+    int x_stride;  // bytes per activation row in shared memory (d * 2 + kMmaRowPad)
+    int w_stride;  // bytes per weight row in shared memory (row bytes + kMmaRowPad)
+    int groups;    // row groups in flight (kMmaGroups bf16, more for the smaller INT4 rows)
 };
+constexpr int kMmaMaxGroups = 8;
 
 // The producer of the tensor-core variant: groups in task order (gate rows of
 // chunk c, then the up rows of chunk c-1), one expect-tx barrier per group.
 template <int NT>
 __device__ void produce_mma(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char* ring, const MmaCfg& mc,
                             int i0, int i1, int n_chunks) {
-    using T = __nv_bfloat16;
-    const unsigned row_bytes = (unsigned)(a.d * sizeof(T));
+    const unsigned row_bytes = (unsigned)a.row_bytes;
+    const unsigned G = (unsigned)mc.groups;
     unsigned grp = 0;
     bool ok = true;
-    auto emit = [&](int kind, int cw, const int* jr, unsigned mask, const T* w) {
-        const unsigned g = grp % kMmaGroups;
-        const unsigned ph = (grp / kMmaGroups) & 1u;
+    auto emit = [&](int kind, int cw, const int* jr, unsigned mask, const unsigned char* w) {
+        const unsigned g = grp % G;
+        const unsigned ph = (grp / G) & 1u;
         if (!wait_or_flag(&sh.empty[g], ph ^ 1u, a.status)) {
             ok = false;
             return;
@@ -752,7 +826,7 @@ __device__ void produce_mma(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
             mbar_arrive_expect_tx(&sh.full[g], (unsigned)__popc(mask) * row_bytes);
             for (unsigned m = mask; m; m &= m - 1u) {
                 const int r = __ffs(m) - 1;
-                tma_load_1d(ring + ((size_t)g * kChunk + r) * mc.row_stride, w + (size_t)jr[r] * a.d, row_bytes,
+                tma_load_1d(ring + ((size_t)g * kChunk + r) * mc.w_stride, w + (size_t)jr[r] * a.row_bytes, row_bytes,
                             &sh.full[g]);
             }
         }
@@ -811,7 +885,7 @@ __device__ void produce_mma(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
                 mbar_arrive(&sh.chunk_free[cw]);
                 mbar_arrive(&sh.gate_ready[cw]);
             } else {
-                emit(kTaskGate, cw, jr, mask, static_cast<const T*>(a.ex[e].wg));
+                emit(kTaskGate, cw, jr, mask, static_cast<const unsigned char*>(a.ex[e].wg));
             }
         }
         if (ok && c >= L) {
@@ -821,19 +895,29 @@ __device__ void produce_mma(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
             if (!ok) break;
             volatile ChunkState<NT>& s = sh.cs[cw];
             const unsigned gm = s.gmask;
-            if (gm) emit(kTaskUp, cw, jr_hist[cw], gm, static_cast<const T*>(a.ex[s.e].wu));
+            if (gm) emit(kTaskUp, cw, jr_hist[cw], gm, static_cast<const unsigned char*>(a.ex[s.e].wu));
         }
     }
     if (ok) emit(kTaskEnd, 0, nullptr, 0u, nullptr);
     // copies in flight must land before the CTA exits
-    for (unsigned q = 0; q < kMmaGroups && q < grp; ++q) {
+    for (unsigned q = 0; q < G && q < grp; ++q) {
         const unsigned gi = grp - 1 - q;
-        if (!wait_or_flag(&sh.full[gi % kMmaGroups], (gi / kMmaGroups) & 1u, a.status)) break;
+        if (!wait_or_flag(&sh.full[gi % G], (gi / G) & 1u, a.status)) break;
     }
 }
 
 // The consumers of the tensor-core variant (C warps, all on every group).
-template <int NT>
+// B fragment pair of two INT4 codes (low nibble = the lower k): bf16x2 of
+// (code - 8), exact. 0x4300 is 128.0 in bf16, whose last mantissa bit is 1.0,
+// so OR-ing a code into it gives 128 + code; subtracting 136 leaves code - 8.
+__device__ __forceinline__ uint32_t q4_pair(uint32_t byte) {
+    const uint32_t v = 0x43004300u | (byte & 0x0Fu) | ((byte & 0xF0u) << 12);
+    __nv_bfloat162 p = *reinterpret_cast<const __nv_bfloat162*>(&v);
+    p = __hsub2(p, __floats2bfloat162_rn(136.0f, 136.0f));
+    return *reinterpret_cast<const uint32_t*>(&p);
+}
+
+template <int NT, bool Q4>
 __device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsigned char* ring,
                             const unsigned char* xb, float* red, const MmaCfg& mc, int cidx, int lane) {
     constexpr int C = GateUpWarps<NT>::C;
@@ -841,7 +925,8 @@ __device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsi
     const int n_ks = a.d / 16;          // K steps of 16
     const int per = n_ks / C;           // even: d % kMmaDAlign == 0
     const int ks0 = cidx * per;
-    const uint32_t x_addr = smem_u32(xb) + (lane % 8) * mc.row_stride + (lane / 8) * 16;
+    const uint32_t x_addr = smem_u32(xb) + (lane % 8) * mc.x_stride + (lane / 8) * 16;
+    const unsigned G = (unsigned)mc.groups;
     // All consumer warps meet at named barriers inside every group, so they
     // must agree on whether to go on: one thread waits, the outcome is shared.
     if (cidx == 0 && lane == 0) {
@@ -854,8 +939,8 @@ __device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsi
         sh.mma_ok = ok;
     }
     for (unsigned grp = 0;; ++grp) {
-        const unsigned g = grp % kMmaGroups;
-        const unsigned parity = (grp / kMmaGroups) & 1u;
+        const unsigned g = grp % G;
+        const unsigned parity = (grp / G) & 1u;
         if (cidx == 0 && lane == 0 && sh.mma_ok) {
             const bool ok = mbar_wait(&sh.full[g], parity);
             if (!ok) atomicOr(a.status, kStatusTimeout);
@@ -867,14 +952,39 @@ __device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsi
         if (!warp_wait(&sh.full[g], parity, lane, a.status)) return;
         const Task tk = sh.task[g];
         if (tk.kind == kTaskEnd) return;
-        const uint32_t w_addr = smem_u32(ring) + (g * kChunk + lane % 8) * mc.row_stride + (lane / 8) * 16;
         float acc0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, acc1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-        for (int ks = ks0; ks < ks0 + per; ks += 2) {
-            uint32_t a0, a2, a0n, a2n, b0, b1, b0n, b1n;
-            ldsm_x4(x_addr + ks * 32, a0, a2, a0n, a2n);
-            ldsm_x4(w_addr + ks * 32, b0, b1, b0n, b1n);
-            mma_bf16_16816(acc0, a0, a2, b0, b1);
-            mma_bf16_16816(acc1, a0n, a2n, b0n, b1n);
+        if constexpr (!Q4) {
+            const uint32_t w_addr = smem_u32(ring) + (g * kChunk + lane % 8) * mc.w_stride + (lane / 8) * 16;
+            for (int ks = ks0; ks < ks0 + per; ks += 2) {
+                uint32_t a0, a2, a0n, a2n, b0, b1, b0n, b1n;
+                ldsm_x4(x_addr + ks * 32, a0, a2, a0n, a2n);
+                ldsm_x4(w_addr + ks * 32, b0, b1, b0n, b1n);
+                mma_bf16_16816(acc0, a0, a2, b0, b1);
+                mma_bf16_16816(acc1, a0n, a2n, b0n, b1n);
+            }
+        } else {
+            // INT4 rows: a K-step pair is one group of 32 codes (16 bytes) and
+            // one binary16 scale per row. Lane (row lane/4, pair lane%4) takes
+            // codes 2t, 2t+1 / 2t+8, 2t+9 of each K-step as its B fragment;
+            // the group's MMA sum is scaled per output column (rows 2t, 2t+1).
+            const int t = lane % 4;
+            const unsigned char* wrow = ring + ((size_t)g * kChunk + lane / 4) * mc.w_stride;
+            const unsigned char* s0row = ring + ((size_t)g * kChunk + 2 * t) * mc.w_stride + a.d / 2;
+            const unsigned char* s1row = s0row + mc.w_stride;
+            for (int ks = ks0; ks < ks0 + per; ks += 2) {
+                uint32_t a0, a2, a0n, a2n;
+                ldsm_x4(x_addr + ks * 32, a0, a2, a0n, a2n);
+                const uint4 cw = lds128(wrow + (size_t)ks * 8);
+                const int sh8 = 8 * t;
+                float dg[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+                mma_bf16_16816(dg, a0, a2, q4_pair((cw.x >> sh8) & 0xFFu), q4_pair((cw.y >> sh8) & 0xFFu));
+                mma_bf16_16816(dg, a0n, a2n, q4_pair((cw.z >> sh8) & 0xFFu), q4_pair((cw.w >> sh8) & 0xFFu));
+                const int grp32 = ks / 2;
+                const float sc0 = __half2float(*reinterpret_cast<const __half*>(s0row + grp32 * 2));
+                const float sc1 = __half2float(*reinterpret_cast<const __half*>(s1row + grp32 * 2));
+                acc0[0] = fmaf(sc0, dg[0], acc0[0]);
+                acc0[1] = fmaf(sc1, dg[1], acc0[1]);
+            }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&sh.empty[g]);
@@ -931,21 +1041,21 @@ __device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsi
     }
 }
 
-template <int NT>
+template <int NT, bool Q4>
 __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_mma(const FfnLaunch a, const MmaCfg mc) {
-    using T = __nv_bfloat16;
+    using T = __nv_bfloat16;  // activations (and bf16 weights)
     constexpr int C = GateUpWarps<NT>::C;
     __shared__ GateUpShared<NT> sh;
     extern __shared__ __align__(128) unsigned char dyn[];
-    unsigned char* xb = dyn;                                       // [8][row_stride] bf16 activations
-    float* red = reinterpret_cast<float*>(dyn + (size_t)kChunk * mc.row_stride);  // [2][C][64]
-    unsigned char* ring = dyn + (size_t)kChunk * mc.row_stride + (size_t)kMmaGroups * C * 64 * sizeof(float);
+    unsigned char* xb = dyn;                                       // [8][x_stride] bf16 activations
+    float* red = reinterpret_cast<float*>(dyn + (size_t)kChunk * mc.x_stride);  // [groups][C][64]
+    unsigned char* ring = dyn + (size_t)kChunk * mc.x_stride + (size_t)mc.groups * C * 64 * sizeof(float);
     const int n_x = a.route ? a.batch : a.nt;
 
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     if (threadIdx.x == 0) {
-        for (int g = 0; g < kMmaGroups; ++g) {
+        for (int g = 0; g < mc.groups; ++g) {
             mbar_init(&sh.full[g], 1);
             mbar_init(&sh.empty[g], C);
         }
@@ -979,7 +1089,7 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_mma(con
     const int x_tok0 = a.route ? 0 : a.tok0;
     // activations as bf16 rows (tokens past the pass are zero)
     for (int t = 0; t < kChunk; ++t) {
-        __nv_bfloat16* xrow = reinterpret_cast<__nv_bfloat16*>(xb + (size_t)t * mc.row_stride);
+        __nv_bfloat16* xrow = reinterpret_cast<__nv_bfloat16*>(xb + (size_t)t * mc.x_stride);
         if (t >= n_x) {
             for (int i = ctid; i < a.d; i += cthreads) xrow[i] = __float2bfloat16_rn(0.0f);
         } else if (a.norm_from_h) {
@@ -1001,18 +1111,31 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_mma(con
         }
     }
     named_bar_sync(1, cthreads);
-    consume_mma<NT>(a, sh, ring, xb, red, mc, warp - 1, lane);
+    consume_mma<NT, Q4>(a, sh, ring, xb, red, mc, warp - 1, lane);
     if constexpr (NT <= kAccMaxTokens) {
         // every chunk is finalized once all consumers are here
         named_bar_sync(1, cthreads);
-        down_partial<T, NT>(a, sh, i0, i1, n_chunks, warp - 1, lane);
+        down_partial<T, NT, Q4>(a, sh, i0, i1, n_chunks, warp - 1, lane);
     }
 }
 
-static size_t mma_smem(int d, MmaCfg* mc) {
-    mc->row_stride = d * 2 + kMmaRowPad;
-    return (size_t)kChunk * mc->row_stride + (size_t)kMmaGroups * GateUpWarps<8>::C * 64 * sizeof(float) +
-           (size_t)kMmaGroups * kChunk * mc->row_stride;
+// Shared memory of the tensor-core variant: activations, the cross-warp
+// sums of every group in flight, and the ring. bf16 rows keep kMmaGroups
+// groups in flight; INT4 rows, 3.6x smaller, as many as fit (up to
+// kMmaMaxGroups) so about as many bytes are in flight.
+static size_t mma_smem(int wdtype, int d, int avail, MmaCfg* mc) {
+    const int row_bytes = wdtype == 2 ? d / 2 + d / 16 : d * 2;
+    mc->x_stride = d * 2 + kMmaRowPad;
+    mc->w_stride = row_bytes + kMmaRowPad;
+    auto bytes = [&](int g) {
+        return (size_t)kChunk * mc->x_stride + (size_t)g * GateUpWarps<8>::C * 64 * sizeof(float) +
+               (size_t)g * kChunk * mc->w_stride;
+    };
+    int g = kMmaGroups;
+    if (wdtype == 2)
+        while (g < kMmaMaxGroups && bytes(g + 1) <= (size_t)avail) ++g;
+    mc->groups = g;
+    return bytes(g);
 }
 
 // ---------------------------------------------------------------------------
@@ -1062,10 +1185,11 @@ static cudaError_t launch_t(const FfnLaunch& a, int grid, cudaStream_t stream, b
     return cudaLaunchKernelEx(&lc, k_gate_up<T, NT>, a, cfg);
 }
 
-template <int NT>
+template <int NT, bool Q4>
 static cudaError_t launch_mma_t(const FfnLaunch& a, int grid, cudaStream_t stream, bool pdl) {
     MmaCfg mc;
-    const size_t smem = mma_smem(a.d, &mc);
+    const size_t smem = mma_smem(Q4 ? 2 : 1, a.d, g_optin - kSmemMargin, &mc);
+    if (smem + kSmemMargin > (size_t)g_optin) return cudaErrorInvalidValue;
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(grid);
     lc.blockDim = dim3(GateUpWarps<NT>::THREADS);
@@ -1076,7 +1200,7 @@ static cudaError_t launch_mma_t(const FfnLaunch& a, int grid, cudaStream_t strea
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = attr;
     lc.numAttrs = pdl ? 1 : 0;
-    return cudaLaunchKernelEx(&lc, k_gate_up_mma<NT>, a, mc);
+    return cudaLaunchKernelEx(&lc, k_gate_up_mma<NT, Q4>, a, mc);
 }
 
 constexpr int kMmaMinTokens = 4;  // narrowest bf16 pass that takes the tensor-core variant
@@ -1084,7 +1208,13 @@ constexpr int kMmaMinTokens = 4;  // narrowest bf16 pass that takes the tensor-c
 static bool use_mma(int wdtype, int d, int pass_tokens) {
     MmaCfg mc;
     return wdtype == 1 && pass_tokens >= kMmaMinTokens && d % kMmaDAlign == 0 &&
-           mma_smem(d, &mc) + kSmemMargin <= (size_t)g_optin;
+           mma_smem(wdtype, d, g_optin - kSmemMargin, &mc) + kSmemMargin <= (size_t)g_optin;
+}
+
+bool int4_supported(int d, int pass_tokens, int optin_smem) {
+    MmaCfg mc;
+    return d % kMmaDAlign == 0 && pass_tokens >= 1 && pass_tokens <= kAccMaxTokens &&
+           mma_smem(2, d, optin_smem - kSmemMargin, &mc) + kSmemMargin <= (size_t)optin_smem;
 }
 
 template <typename T, int NT>
@@ -1107,24 +1237,30 @@ cudaError_t prepare_gate_up(int optin_smem) {
     if (e == cudaSuccess) e = prepare_t<float, 2>(optin_smem);
     if (e == cudaSuccess) e = prepare_t<float, 4>(optin_smem);
     if (e == cudaSuccess) e = prepare_t<float, 8>(optin_smem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_gate_up_mma<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin_smem - kSmemMargin);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_gate_up_mma<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin_smem - kSmemMargin);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_gate_up_mma<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin_smem - kSmemMargin);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_gate_up_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin_smem - kSmemMargin);
+    const int dyn = optin_smem - kSmemMargin;
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<4, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<8, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     return e;
 }
 
 cudaError_t launch_gate_up(const FfnLaunch& a, int wdtype, int pass_tokens, int grid,
                            cudaStream_t stream, bool pdl) {
+    if (wdtype == 2) {
+        // INT4 rows: the tensor-core variant, passes of 1-2 tokens
+        if (a.d % kMmaDAlign != 0) return cudaErrorInvalidValue;
+        if (pass_tokens == 1) return launch_mma_t<1, true>(a, grid, stream, pdl);
+        if (pass_tokens == 2) return launch_mma_t<2, true>(a, grid, stream, pdl);
+        return cudaErrorInvalidValue;
+    }
     if (use_mma(wdtype, a.d, pass_tokens)) {
-        if (pass_tokens == 1) return launch_mma_t<1>(a, grid, stream, pdl);
-        if (pass_tokens == 2) return launch_mma_t<2>(a, grid, stream, pdl);
-        if (pass_tokens == 4) return launch_mma_t<4>(a, grid, stream, pdl);
-        if (pass_tokens == 8) return launch_mma_t<8>(a, grid, stream, pdl);
+        if (pass_tokens == 1) return launch_mma_t<1, false>(a, grid, stream, pdl);
+        if (pass_tokens == 2) return launch_mma_t<2, false>(a, grid, stream, pdl);
+        if (pass_tokens == 4) return launch_mma_t<4, false>(a, grid, stream, pdl);
+        if (pass_tokens == 8) return launch_mma_t<8, false>(a, grid, stream, pdl);
     }
     if (wdtype == 1) {
         switch (pass_tokens) {

@@ -49,7 +49,8 @@ struct ExpertPtrs {
 // pass's tokens tok0 .. tok0+nt-1 with weight 1.
 struct FfnLaunch {
     int d, m;
-    int elem_bytes;         // bytes per weight element (2 bf16, 4 fp32)
+    int elem_bytes;         // bytes per weight element (2 bf16, 4 fp32; 0 for INT4 rows)
+    int row_bytes;          // bytes per weight row (d * elem_bytes, or 9d/16 for INT4)
     int n_rows;             // size of the row space: m, or the list length
     const int32_t* rows;    // predictor list (ascending neuron ids) or nullptr
     int batch;              // tokens of the whole call
@@ -346,4 +347,6 @@ cudaError_t prepare_router();
 // shared memory; -1 if fewer than 4 row slots fit.
 int gate_up_config(int wdtype, int d, int x_tokens, int optin_smem, int* slots, int* slot_bytes,
                    int* xs_stride, size_t* smem);
+// Whether INT4 rows of d weights can run passes of `pass_tokens` tokens.
+bool int4_supported(int d, int pass_tokens, int optin_smem);
 }  // namespace tsffn

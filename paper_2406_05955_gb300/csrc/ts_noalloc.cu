@@ -132,6 +132,7 @@ extern "C" ts_status ts_ffn_forward_noalloc(int d, int m, ts_dtype wdtype, const
     a.d = d;
     a.m = m;
     a.elem_bytes = elem;
+    a.row_bytes = d * elem;
     a.rows = active_idx;
     a.n_rows = active_idx ? n_active : m;
     a.batch = batch;
