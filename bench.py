@@ -179,16 +179,29 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # workload set-up
 # ---------------------------------------------------------------------------
-def make_stack(ts, wl, dev, batch: int, predictor: bool, n_layers: int | None = None):
-    cfg = dict(wl.WORKLOADS["mistral7b-ffn-stack-bf16-predictor" if predictor
-                            else "mistral7b-ffn-stack-bf16-b1-act10"])
+def stack_workload(args) -> str:
+    if args.workload == "predictor":
+        return "mistral7b-ffn-stack-bf16-predictor"
+    if args.workload == "int4":
+        return "mistral7b-ffn-stack-int4-b1-act10"
+    return "mistral7b-ffn-stack-bf16-b1-act10"
+
+
+def make_stack(ts, wl, dev, batch: int, predictor: bool, n_layers: int | None = None, name: str | None = None):
+    cfg = dict(wl.WORKLOADS[name or ("mistral7b-ffn-stack-bf16-predictor" if predictor
+                                     else "mistral7b-ffn-stack-bf16-b1-act10")])
     if n_layers:
         cfg["layers"] = n_layers
     d, m, n_layers = cfg["d"], cfg["m"], cfg["layers"]
+    int4 = cfg["dtype"] == "int4"
     layers, ffns, lists = [], [], []
     for l in range(n_layers):
-        L = wl.ffn_layer(d, m, activation=cfg["activation"], dtype=torch.bfloat16,
-                         seed=wl.layer_seed(cfg["seed"], l), device=dev)
+        if int4:
+            L = wl.ffn_layer_int4(d, m, activation=cfg["activation"], seed=wl.layer_seed(cfg["seed"], l),
+                                  device=dev)
+        else:
+            L = wl.ffn_layer(d, m, activation=cfg["activation"], dtype=torch.bfloat16,
+                             seed=wl.layer_seed(cfg["seed"], l), device=dev)
         layers.append(L)
         ffns.append(ts.Ffn(L.w_gate, L.w_up, L.w_down, max_batch=batch))
         if predictor:
@@ -197,14 +210,22 @@ def make_stack(ts, wl, dev, batch: int, predictor: bool, n_layers: int | None = 
     return cfg, layers, ffns, (lists if predictor else None)
 
 
-def needed_bytes_stack(ffns, lists, elem=2) -> dict:
+def row_bytes(f) -> int:
+    """Bytes of one weight row of an Ffn handle (bf16, fp32 or INT4 rows)."""
+    if f.wcode == 2:
+        return f.d // 2 + f.d // 16
+    return f.d * (2 if f.dtype == torch.bfloat16 else 4)
+
+
+def needed_bytes_stack(ffns, lists) -> dict:
     """Per-layer algorithmic bytes from the last forward's active sets (union over the batch)."""
     tot_gate_up, tot_down, per = 0, 0, []
     for l, f in enumerate(ffns):
         g, b = f.get_active(-1)
         n_rows = f.m if lists is None else int(lists[l].numel())
-        gate_kernel = (n_rows + len(g)) * f.d * elem  # gate rows + gathered up rows
-        down_kernel = len(b) * f.d * elem
+        rb = row_bytes(f)
+        gate_kernel = (n_rows + len(g)) * rb  # gate rows + gathered up rows
+        down_kernel = len(b) * rb
         tot_gate_up += gate_kernel
         tot_down += down_kernel
         per.append((len(g), len(b)))
@@ -310,7 +331,8 @@ def run_ours(args, dist: Dist) -> dict | None:
     torch.cuda.set_device(dev)
     B = args.batch
     predictor = args.workload == "predictor"
-    cfg, layers, ffns, lists = make_stack(ts, wl, dev, B, predictor, args.layers)
+    int4 = args.workload == "int4"
+    cfg, layers, ffns, lists = make_stack(ts, wl, dev, B, predictor, args.layers, name=stack_workload(args))
     n_layers = cfg["layers"]
     h0 = wl.residual(B, cfg["d"], seed=cfg["seed"] - 1, device=dev)
     h = h0.clone()
@@ -353,7 +375,7 @@ def run_ours(args, dist: Dist) -> dict | None:
            "h2d_bytes_per_step": h_host.numel() * 4, "d2h_bytes_per_step": out_host.numel() * 4}
 
     # dominant kernel: gate+up, timed alone per layer
-    x = wl.tokens(B, cfg["d"], dtype=torch.bfloat16, seed=5, device=dev)
+    x = wl.tokens(B, cfg["d"], dtype=torch.bfloat16, seed=5, device=dev)  # bf16 activations (INT4 too)
     graph.launch(stream)
     torch.cuda.synchronize()
     nb = needed_bytes_stack(ffns, lists)
@@ -369,12 +391,12 @@ def run_ours(args, dist: Dist) -> dict | None:
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": ("mistral7b-ffn-stack-bf16-predictor" if predictor
-                                else "mistral7b-ffn-stack-bf16-b1-act10"),
+        "vs_baseline": None, "dtype": "int4 weights, bf16 activations, fp32 accumulate" if int4 else "bf16",
+        "data": "synthetic",
+        "config": {"workload": stack_workload(args),
                    "d": cfg["d"], "m": cfg["m"], "layers": n_layers, "batch": B,
-                   "activation": cfg["activation"], "weights_gb": round(3 * cfg["d"] * cfg["m"] * 2 * n_layers / 1e9, 2),
-                   "l2": f"no flush: the {3 * cfg['d'] * cfg['m'] * 2 * n_layers / 1e9:.2f} GB of weights "
+                   "activation": cfg["activation"], "weights_gb": round(3 * cfg["m"] * row_bytes(ffns[0]) * n_layers / 1e9, 2),
+                   "l2": f"no flush: the {3 * cfg['m'] * row_bytes(ffns[0]) * n_layers / 1e9:.2f} GB of weights "
                          "streamed per step exceed the 129 MB L2",
                    "parallelism": f"replicas x{dist.world}"},
         "layers_per_s": value * n_layers / B,
@@ -391,17 +413,17 @@ def run_ours(args, dist: Dist) -> dict | None:
                                 "down projection)" if B <= 2 else "k_gate_up (gate GEMV + gathered up projection)"),
                      "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                      "frac": achieved / peaks["hbm_gbs"], "peak_source": peaks["source"],
-                     "traffic": None if predictor or B != 1 else ncu_traffic(),
+                     "traffic": None if predictor or int4 or B != 1 else ncu_traffic(),
                      "bytes_per_launch": gate_up_bytes,
                      "avg_launch_us": t_gate_up * 1e6},
         "e2e": e2e,
         "gpu_launches": 2 * n_layers * args.steps * ((B + 7) // 8),
         "clocks": clk,
     }
-    if not args.no_dense:
+    if not args.no_dense and not int4:
         result["dense_cublas"] = {"value": dense_cublas_tokens_per_s(layers, B, dev), "unit": UNIT,
                                   "what": "same weights, dense ReLU-gated FFN via torch.matmul (cuBLAS), graph-replayed"}
-    if dist.rank == 0 and not args.no_cpu_baseline:
+    if dist.rank == 0 and not args.no_cpu_baseline and not int4:
         result["cpu_baseline"] = cpu_baseline(layers, lists, B, n_layers)
     for f in ffns:
         f.close()
@@ -427,16 +449,21 @@ def run_moe(args, dist: Dist) -> dict:
     import paper_2406_05955_gb300 as ts
     from paper_2406_05955_gb300 import workload as wl
 
-    name = "mixtral47b-moe-stack-bf16-top2"
+    name = "mixtral47b-moe-stack-int4-top2" if args.workload == "moe-int4" else "mixtral47b-moe-stack-bf16-top2"
     cfg = wl.WORKLOADS[name]
+    int4 = cfg["dtype"] == "int4"
     dev = torch.device("cuda", dist.local)
     torch.cuda.set_device(dev)
     B, d, m, E, k = args.batch, cfg["d"], cfg["m"], cfg["experts"], cfg["top_k"]
     n_layers = args.layers or cfg["layers"]
     experts, moes = [], []
     for l in range(n_layers):
-        ex = [wl.ffn_layer(d, m, activation=cfg["activation"], dtype=torch.bfloat16,
-                           seed=wl.layer_seed(cfg["seed"], l, e), device=dev) for e in range(E)]
+        if int4:
+            ex = [wl.ffn_layer_int4(d, m, activation=cfg["activation"], seed=wl.layer_seed(cfg["seed"], l, e),
+                                    device=dev) for e in range(E)]
+        else:
+            ex = [wl.ffn_layer(d, m, activation=cfg["activation"], dtype=torch.bfloat16,
+                               seed=wl.layer_seed(cfg["seed"], l, e), device=dev) for e in range(E)]
         ffns = [ts.Ffn(L.w_gate, L.w_up, L.w_down, max_batch=B) for L in ex]
         wr = wl.router(E, d, seed=wl.layer_seed(cfg["seed"], l) + 99, device=dev)
         experts.append((ex, ffns, wr))
@@ -458,16 +485,17 @@ def run_moe(args, dist: Dist) -> dict:
         sel, _ = mo.get_routing(B)
         for e in sorted(set(sel.ravel().tolist())):
             g, b = mo.get_active(e, -1)
-            need += (m + len(g) + len(b)) * d * 2
+            need += (m + len(g) + len(b)) * row_bytes(mo.experts[e])
     peaks = load_peaks()
     step_s = t_max / args.steps
     res = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "vs_baseline": None, "dtype": "int4 weights, bf16 activations, fp32 accumulate" if int4 else "bf16",
+        "data": "synthetic",
         "config": {"workload": name, "d": d, "m": m, "experts": E, "top_k": k, "layers": n_layers, "batch": B,
                    "activation": cfg["activation"],
-                   "weights_gb": round(E * 3 * d * m * 2 * n_layers / 1e9, 1),
+                   "weights_gb": round(E * 3 * m * row_bytes(experts[0][1][0]) * n_layers / 1e9, 1),
                    "l2": "no flush: the experts streamed per step exceed the 129 MB L2",
                    "parallelism": f"replicas x{dist.world}"},
         "needed_bytes_roofline": {"bytes_per_token": need / B, "achieved_gbs": need / step_s / 1e9,
@@ -580,7 +608,7 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["stack", "predictor", "moe", "sweep"], default="stack")
+    ap.add_argument("--workload", choices=["stack", "predictor", "moe", "sweep", "int4", "moe-int4"], default="stack")
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--layers", type=int, default=0,
                     help="fewer layers than the workload's 32 (profiling cases only; not a bench line)")
@@ -601,7 +629,7 @@ def main():
             if dist.rank == 0:
                 build()
             dist.barrier()
-            if args.workload == "moe":
+            if args.workload in ("moe", "moe-int4"):
                 res = run_moe(args, dist)
             elif args.workload == "sweep":
                 res = run_sweep(args, dist)

@@ -797,9 +797,11 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint3
 }
 
 struct MmaCfg {
-    int x_stride;  // bytes per activation row in shared memory (d * 2 + kMmaRowPad)
-    int w_stride;  // bytes per weight row in shared memory (row bytes + kMmaRowPad)
-    int groups;    // row groups in flight (kMmaGroups bf16, more for the smaller INT4 rows)
+    int x_stride;   // bytes per activation row in shared memory (d * 2 + kMmaRowPad)
+    int w_stride;   // bytes per weight row in shared memory (row bytes + kMmaRowPad)
+    int groups;     // row groups in flight (kMmaGroups bf16, more for the smaller INT4 rows)
+    int lookahead;  // gate groups issued ahead of their chunk's up group
+    int end_tasks;  // end groups to emit: 1 (all consumers read each group) or one per consumer
 };
 constexpr int kMmaMaxGroups = 8;
 
@@ -833,7 +835,7 @@ __device__ void produce_mma(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
         ++grp;
     };
     const int n_local = i1 - i0;
-    constexpr int L = 1;  // gate groups ahead of their up group
+    const int L = mc.lookahead;  // gate groups ahead of their up group
     int jr_hist[kWindow][kChunk];
     for (int c = 0; ok && c < n_local + L; ++c) {
         if (c < n_local) {
@@ -898,7 +900,7 @@ __device__ void produce_mma(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
             if (gm) emit(kTaskUp, cw, jr_hist[cw], gm, static_cast<const unsigned char*>(a.ex[s.e].wu));
         }
     }
-    if (ok) emit(kTaskEnd, 0, nullptr, 0u, nullptr);
+    for (int q = 0; q < mc.end_tasks && ok; ++q) emit(kTaskEnd, 0, nullptr, 0u, nullptr);
     // copies in flight must land before the CTA exits
     for (unsigned q = 0; q < G && q < grp; ++q) {
         const unsigned gi = grp - 1 - q;
@@ -1135,7 +1137,188 @@ static size_t mma_smem(int wdtype, int d, int avail, MmaCfg* mc) {
     if (wdtype == 2)
         while (g < kMmaMaxGroups && bytes(g + 1) <= (size_t)avail) ++g;
     mc->groups = g;
+    mc->lookahead = 1;
+    mc->end_tasks = 1;
     return bytes(g);
+}
+
+// ---------------------------------------------------------------------------
+// INT4 rows, passes of 1-2 tokens: each consumer warp takes whole groups (a
+// chunk's 8 gate rows, or its gate-active up rows) over the full K, so no
+// warp waits on another: INT4 rows are 3.6x smaller than bf16 rows, and the
+// shared-group design above would spend more time in its per-group barriers
+// than in the MMAs. Consumer warp c owns ring slot c (one group each).
+// ---------------------------------------------------------------------------
+constexpr int kQ4Lookahead = 5;  // gate groups ahead of their up group (< kWindow)
+
+template <int NT>
+__device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, const unsigned char* ring,
+                            const unsigned char* xb, const MmaCfg& mc, int cidx, int lane) {
+    constexpr int C = GateUpWarps<NT>::C;
+    const int d = a.d;
+    const int t = lane % 4;
+    const uint32_t x_addr = smem_u32(xb) + (lane % 8) * mc.x_stride + (lane / 8) * 16;
+    const unsigned slot = (unsigned)cidx;  // groups == C: this warp's only slot
+    unsigned phase = 0;
+    if (a.test_stall && cidx == 0) {
+        // the failure-detection test: a wait that can only run out
+        if (!warp_wait(&sh.never, 0u, lane, a.status)) return;
+    }
+    for (;;) {
+        if (!warp_wait(&sh.full[slot], phase, lane, a.status)) return;
+        phase ^= 1u;
+        const Task tk = sh.task[slot];
+        if (tk.kind == kTaskEnd) return;
+        const unsigned char* base = ring + (size_t)slot * kChunk * mc.w_stride;
+        const unsigned char* wrow = base + (size_t)(lane / 4) * mc.w_stride;
+        const unsigned char* s0row = base + (size_t)(2 * t) * mc.w_stride + d / 2;
+        const unsigned char* s1row = s0row + mc.w_stride;
+        float v0a = 0.0f, v1a = 0.0f, v0b = 0.0f, v1b = 0.0f;  // two chains (even / odd groups)
+        const int sh8 = 8 * t;
+        for (int gq = 0; gq < d / 32; gq += 2) {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int ks = 2 * (gq + h);
+                uint32_t a0, a2, a0n, a2n;
+                ldsm_x4(x_addr + ks * 32, a0, a2, a0n, a2n);
+                const uint4 cw = lds128(wrow + (size_t)ks * 8);
+                float dg[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+                mma_bf16_16816(dg, a0, a2, q4_pair((cw.x >> sh8) & 0xFFu), q4_pair((cw.y >> sh8) & 0xFFu));
+                mma_bf16_16816(dg, a0n, a2n, q4_pair((cw.z >> sh8) & 0xFFu), q4_pair((cw.w >> sh8) & 0xFFu));
+                const float sc0 = __half2float(*reinterpret_cast<const __half*>(s0row + (gq + h) * 2));
+                const float sc1 = __half2float(*reinterpret_cast<const __half*>(s1row + (gq + h) * 2));
+                if (h == 0) {
+                    v0a = fmaf(sc0, dg[0], v0a);
+                    v1a = fmaf(sc1, dg[1], v1a);
+                } else {
+                    v0b = fmaf(sc0, dg[0], v0b);
+                    v1b = fmaf(sc1, dg[1], v1b);
+                }
+            }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sh.empty[slot]);
+        // D row = token lane/4, columns = rows 2t, 2t+1 of the group
+        volatile ChunkState<NT>& s = sh.cs[tk.cw];
+        const int e = s.e;
+        const int ntok = sh.es.ntok[e];
+        const int tok = lane / 4;
+        const float v[2] = {v0a + v0b, v1a + v1b};
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const int r = 2 * t + q;
+            if ((tk.r >> r) & 1) {
+#pragma unroll
+                for (int k = 0; k < NT; ++k) {
+                    const int tk_x = a.route ? sh.es.tok[e][k] : k;
+                    if (k < ntok && tk_x == tok) {
+                        if (tk.kind == kTaskGate)
+                            s.g[r][k] = v[q];
+                        else
+                            s.u[r][k] = v[q];
+                    }
+                }
+            }
+        }
+        __syncwarp();
+        __threadfence_block();
+        if (tk.kind == kTaskGate) {
+            bool ga = false;
+            if (lane < kChunk && s.jr[lane] >= 0) {
+#pragma unroll
+                for (int k = 0; k < NT; ++k) ga |= (k < ntok) && (s.g[lane][k] > 0.0f);
+            }
+            const unsigned gm = __ballot_sync(0xffffffffu, ga);
+            if (lane == 0) s.gmask = gm;
+            __syncwarp();
+            __threadfence_block();
+            if (gm == 0u) finalize_chunk<NT>(a, sh, tk.cw, lane);
+            if (lane == 0) mbar_arrive(&sh.gate_ready[tk.cw]);
+        } else {
+            finalize_chunk<NT>(a, sh, tk.cw, lane);
+        }
+    }
+}
+
+template <int NT>
+__global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(const FfnLaunch a, const MmaCfg mc) {
+    using T = __nv_bfloat16;  // activations
+    constexpr int C = GateUpWarps<NT>::C;
+    __shared__ GateUpShared<NT> sh;
+    extern __shared__ __align__(128) unsigned char dyn[];
+    unsigned char* xb = dyn;                                     // [8][x_stride] bf16 activations
+    unsigned char* ring = dyn + (size_t)kChunk * mc.x_stride;    // [C][8][w_stride]
+    const int n_x = a.route ? a.batch : a.nt;
+
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    if (threadIdx.x == 0) {
+        for (int g = 0; g < mc.groups; ++g) {
+            mbar_init(&sh.full[g], 1);
+            mbar_init(&sh.empty[g], 1);
+        }
+        mbar_init(&sh.never, 1);
+        for (int q = 0; q < kMaxLocal; ++q) sh.pd.ub[q] = 0;
+        for (int w = 0; w < kWindow; ++w) {
+            mbar_init(&sh.gate_ready[w], 1);
+            mbar_init(&sh.chunk_free[w], 1);
+        }
+        mbar_fence_init();
+    }
+    const bool early = a.rows == nullptr && a.route == nullptr;
+    if (!early) pdl_wait();
+    resolve_experts(a, sh.es);
+    pdl_launch_dependents();
+
+    const int n_chunks = (a.n_rows + kChunk - 1) / kChunk;
+    const int n_items = sh.es.n_act * n_chunks;
+    const int i0 = (int)((long long)n_items * blockIdx.x / gridDim.x);
+    const int i1 = (int)((long long)n_items * (blockIdx.x + 1) / gridDim.x);
+
+    if (warp == 0) {
+        if (lane == 0) produce_mma<NT>(a, sh, ring, mc, i0, i1, n_chunks);
+        return;
+    }
+    if (early) pdl_wait();
+    const int ctid = threadIdx.x - kWarp;
+    const int cthreads = C * kWarp;
+    const int x_tok0 = a.route ? 0 : a.tok0;
+    for (int t = 0; t < kChunk; ++t) {
+        __nv_bfloat16* xrow = reinterpret_cast<__nv_bfloat16*>(xb + (size_t)t * mc.x_stride);
+        if (t >= n_x) {
+            for (int i = ctid; i < a.d; i += cthreads) xrow[i] = __float2bfloat16_rn(0.0f);
+        } else if (a.norm_from_h) {
+            const float* hr = a.h + (size_t)(x_tok0 + t) * a.d;
+            float ss = 0.0f;
+            for (int i = ctid; i < a.d; i += cthreads) ss = fmaf(hr[i], hr[i], ss);
+            ss = warp_sum(ss);
+            if (lane == 0) sh.red[warp - 1] = ss;
+            named_bar_sync(1, cthreads);
+            float tot = 0.0f;
+            for (int w = 0; w < C; ++w) tot += sh.red[w];
+            const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)a.d), 1e-5f));
+            for (int i = ctid; i < a.d; i += cthreads)
+                xrow[i] = __float2bfloat16_rn((i == a.d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hr[i], rms)));
+            named_bar_sync(1, cthreads);
+        } else {
+            const T* xr = static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d;
+            for (int i = ctid; i < a.d; i += cthreads) xrow[i] = xr[i];
+        }
+    }
+    named_bar_sync(1, cthreads);
+    consume_q4w<NT>(a, sh, ring, xb, mc, warp - 1, lane);
+    // every chunk is finalized once all consumers are here
+    named_bar_sync(1, cthreads);
+    down_partial<T, NT, true>(a, sh, i0, i1, n_chunks, warp - 1, lane);
+}
+
+static size_t q4w_smem(int d, MmaCfg* mc) {
+    mc->x_stride = d * 2 + kMmaRowPad;
+    mc->w_stride = d / 2 + d / 16 + kMmaRowPad;
+    mc->groups = GateUpWarps<1>::C;
+    mc->lookahead = kQ4Lookahead;
+    mc->end_tasks = GateUpWarps<1>::C;
+    return (size_t)kChunk * mc->x_stride + (size_t)mc->groups * kChunk * mc->w_stride;
 }
 
 // ---------------------------------------------------------------------------
@@ -1203,6 +1386,24 @@ static cudaError_t launch_mma_t(const FfnLaunch& a, int grid, cudaStream_t strea
     return cudaLaunchKernelEx(&lc, k_gate_up_mma<NT, Q4>, a, mc);
 }
 
+template <int NT>
+static cudaError_t launch_q4w_t(const FfnLaunch& a, int grid, cudaStream_t stream, bool pdl) {
+    MmaCfg mc;
+    const size_t smem = q4w_smem(a.d, &mc);
+    if (smem + kSmemMargin > (size_t)g_optin) return cudaErrorInvalidValue;
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(GateUpWarps<NT>::THREADS);
+    lc.dynamicSmemBytes = smem;
+    lc.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&lc, k_gate_up_q4w<NT>, a, mc);
+}
+
 constexpr int kMmaMinTokens = 4;  // narrowest bf16 pass that takes the tensor-core variant
 
 static bool use_mma(int wdtype, int d, int pass_tokens) {
@@ -1214,7 +1415,7 @@ static bool use_mma(int wdtype, int d, int pass_tokens) {
 bool int4_supported(int d, int pass_tokens, int optin_smem) {
     MmaCfg mc;
     return d % kMmaDAlign == 0 && pass_tokens >= 1 && pass_tokens <= kAccMaxTokens &&
-           mma_smem(2, d, optin_smem - kSmemMargin, &mc) + kSmemMargin <= (size_t)optin_smem;
+           q4w_smem(d, &mc) + kSmemMargin <= (size_t)optin_smem;
 }
 
 template <typename T, int NT>
@@ -1242,18 +1443,18 @@ cudaError_t prepare_gate_up(int optin_smem) {
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<4, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<8, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_q4w<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_q4w<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     return e;
 }
 
 cudaError_t launch_gate_up(const FfnLaunch& a, int wdtype, int pass_tokens, int grid,
                            cudaStream_t stream, bool pdl) {
     if (wdtype == 2) {
-        // INT4 rows: the tensor-core variant, passes of 1-2 tokens
+        // INT4 rows: tensor cores, one group per warp, passes of 1-2 tokens
         if (a.d % kMmaDAlign != 0) return cudaErrorInvalidValue;
-        if (pass_tokens == 1) return launch_mma_t<1, true>(a, grid, stream, pdl);
-        if (pass_tokens == 2) return launch_mma_t<2, true>(a, grid, stream, pdl);
+        if (pass_tokens == 1) return launch_q4w_t<1>(a, grid, stream, pdl);
+        if (pass_tokens == 2) return launch_q4w_t<2>(a, grid, stream, pdl);
         return cudaErrorInvalidValue;
     }
     if (use_mma(wdtype, a.d, pass_tokens)) {

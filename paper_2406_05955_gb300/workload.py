@@ -196,6 +196,13 @@ WORKLOADS = {
         d=MISTRAL_D, m=MISTRAL_M, dtype="bf16", experts=8, top_k=2, batches=(1, 8), layers=N_LAYERS,
         activation=0.20, seed=3000,
         desc="32-layer Mixtral-shaped MoE, 8 experts, top-2, ~20% combined activation per expert"),
+    "mistral7b-ffn-stack-int4-b1-act10": dict(
+        d=MISTRAL_D, m=MISTRAL_M, dtype="int4", batch=1, layers=N_LAYERS, activation=0.10, seed=1000,
+        desc="the batch-1 Mistral-shaped stack with INT4 rows (4-bit codes, binary16 scale per 32)"),
+    "mixtral47b-moe-stack-int4-top2": dict(
+        d=MISTRAL_D, m=MISTRAL_M, dtype="int4", experts=8, top_k=2, batches=(1,), layers=N_LAYERS,
+        activation=0.20, seed=3000,
+        desc="the Mixtral-shaped MoE stack with INT4 experts (the paper's Mixtral-47B-INT4 setting)"),
     "mistral7b-ffn-stack-bf16-predictor": dict(
         d=MISTRAL_D, m=MISTRAL_M, dtype="bf16", batch=1, layers=N_LAYERS, activation=0.10,
         list_len=1434, zipf_s=1.1, seed=1000,
