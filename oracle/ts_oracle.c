@@ -32,9 +32,11 @@
  * upper 16 bits of an IEEE binary32), decoded exactly to double. Weights may
  * also be stored as INT4 groups (the weight-only 4-bit storage of the paper's
  * Mixtral-47B-INT4 rows, Tables 7-9): per neuron row of d weights, d/2 bytes
- * of 4-bit codes (element i in byte i/2, low nibble for even i) followed by
- * d/32 IEEE binary16 scales, one per group of 32 consecutive elements; the
- * weight is scale * (code - 8), decoded exactly to double.
+ * of 4-bit codes followed by d/32 IEEE binary16 scales, one per group of 32
+ * consecutive elements; the weight is scale * (code - 8), decoded exactly to
+ * double. A group's 16 code bytes are four little-endian 32-bit words;
+ * element e = 8s + 2t + h (s, t in 0..3, h in 0..1) of the group is the
+ * nibble s + 4h of word t.
  */
 #include <math.h>
 #include <stdint.h>
@@ -73,7 +75,10 @@ static double welem(const void* base, int wdtype, int d, int j, int i) {
         return (double)f;
     }
     const uint8_t* row = (const uint8_t*)base + (size_t)j * int4_row_bytes(d);
-    const int code = (row[i / 2] >> (4 * (i & 1))) & 15;
+    const int e = i % 32, s = e / 8, t = (e % 8) / 2, hh = e % 2;
+    const int nib = s + 4 * hh; /* nibble of word t */
+    const uint8_t byte = row[(size_t)(i / 32) * 16 + 4 * t + nib / 2];
+    const int code = (byte >> (4 * (nib % 2))) & 15;
     const uint8_t* sp = row + d / 2 + (size_t)(i / 32) * 2;
     const uint16_t h = (uint16_t)(sp[0] | (sp[1] << 8)); /* little-endian */
     return half_to_double(h) * (double)(code - 8);

@@ -84,10 +84,12 @@ def ffn_layer(d: int, m: int, *, activation: float = 0.10, mu: float | None = No
 
 # ---------------------------------------------------------------------------
 # INT4 weight storage (the weight-only 4-bit rows of the paper's INT4 models,
-# Tables 7-9): per neuron row of d weights, d/2 bytes of 4-bit codes (element
-# i in byte i/2, low nibble for even i) followed by d/32 IEEE binary16 scales
-# (little-endian), one per group of 32 consecutive elements. A stored weight
-# is scale * (code - 8).
+# Tables 7-9): per neuron row of d weights, d/2 bytes of 4-bit codes followed
+# by d/32 IEEE binary16 scales (little-endian), one per group of 32
+# consecutive elements. A stored weight is scale * (code - 8). Within a
+# group's 16 code bytes, read as four little-endian 32-bit words, element
+# e = 8s + 2t + h (s, t in 0..3, h in 0..1) sits in word t at nibble s + 4h
+# (bits 4(s+4h) .. 4(s+4h)+3).
 # ---------------------------------------------------------------------------
 INT4_GROUP = 32
 
@@ -108,9 +110,14 @@ def quantize_int4(w: torch.Tensor) -> torch.Tensor:
     wf = w.detach().float().reshape(m, d // INT4_GROUP, INT4_GROUP)
     scale = (wf.abs().amax(-1) / 7.0).to(torch.float16)
     scale = torch.where(scale == 0, torch.ones_like(scale), scale)
-    q = torch.clamp(torch.round(wf / scale.float().unsqueeze(-1)), -8, 7).to(torch.int32) + 8
-    q = q.reshape(m, d)
-    codes = (q[:, 0::2] | (q[:, 1::2] << 4)).to(torch.uint8)
+    q = torch.clamp(torch.round(wf / scale.float().unsqueeze(-1)), -8, 7).to(torch.int64) + 8  # [m][G][32]
+    # element e = 8s + 2t + h -> word t, nibble s + 4h
+    q = q.reshape(m, d // INT4_GROUP, 4, 4, 2)          # [m][G][s][t][h]
+    shifts = 4 * (torch.arange(4, device=w.device).view(4, 1, 1) +
+                  4 * torch.arange(2, device=w.device).view(1, 1, 2))  # [s][1][h]
+    words = (q << shifts).sum(dim=(2, 4))               # [m][G][t], disjoint nibbles
+    codes = torch.stack([(words >> (8 * b)) & 0xFF for b in range(4)], dim=-1).to(torch.uint8)
+    codes = codes.reshape(m, d // 2)
     scales = scale.contiguous().view(torch.uint8).reshape(m, (d // INT4_GROUP) * 2)
     return torch.cat([codes, scales], dim=1).contiguous()
 

@@ -1,14 +1,17 @@
 """Pins for the oracle's INT4 weight storage (the 4-bit weight-only rows of the
 paper's INT4 models, Tables 7-9), against things other than the oracle.
 
-Row layout: d/2 bytes of 4-bit codes (element i in byte i/2, low nibble for
-even i), then d/32 little-endian IEEE binary16 scales; weight = scale * (code - 8).
+Row layout: d/2 bytes of 4-bit codes, then d/32 little-endian IEEE binary16
+scales; weight = scale * (code - 8). A group of 32 elements owns 16 code bytes,
+read as four little-endian 32-bit words: element e = 8s + 2t + h (s, t in
+0..3, h in 0..1) is nibble s + 4h of word t.
 Pinned by: a hand-worked FFN whose codes and scales were chosen so every value
 is exact; binary16 special cases against numpy's float16 decoding; random
 layers against an independent numpy decoding followed by library matmuls; the
 all-active case as a plain ReGLU FFN; and mistakes planted in a CPU
-restatement of the decoding (swapped nibbles, offset 7, a shifted scale group,
-big-endian scales), which the pins reject.
+restatement of the decoding (the two halves of a word swapped, plain sequential
+nibbles, offset 7, a shifted scale group, big-endian scales), which the pins
+reject.
 """
 import numpy as np
 import pytest
@@ -19,14 +22,44 @@ from paper_2406_05955_gb300 import workload as wl
 D = 32  # one group per row
 
 
+def _pack(c: np.ndarray) -> np.ndarray:
+    """Code bytes of one row of d codes: per group of 32, word t holds element
+    8s + 2t + h at nibble s + 4h; words stored little-endian."""
+    out = []
+    for g in range(len(c) // 32):
+        grp = c[32 * g: 32 * g + 32]
+        for t in range(4):
+            word = 0
+            for s_ in range(4):
+                for h in range(2):
+                    word |= int(grp[8 * s_ + 2 * t + h]) << (4 * (s_ + 4 * h))
+            out += [(word >> (8 * b)) & 0xFF for b in range(4)]
+    return np.array(out, np.uint8)
+
+
+def _unpack(q: np.ndarray, d: int, halves=(0, 1), sequential=False) -> np.ndarray:
+    """Codes [rows][d] from the code bytes of each row (the inverse of _pack)."""
+    b = q[:, : d // 2].astype(np.int64)
+    codes = np.empty((q.shape[0], d), np.int64)
+    if sequential:  # a planted mistake: element i in byte i/2, low nibble for even i
+        codes[:, 0::2], codes[:, 1::2] = b & 0x0F, b >> 4
+        return codes
+    words = b.reshape(q.shape[0], d // 32, 4, 4)
+    words = words[..., 0] | (words[..., 1] << 8) | (words[..., 2] << 16) | (words[..., 3] << 24)
+    for s_ in range(4):
+        for t in range(4):
+            for h in range(2):
+                codes[:, 8 * s_ + 2 * t + h::32] = (words[:, :, t] >> (4 * (s_ + 4 * halves[h]))) & 0xF
+    return codes
+
+
 def _row(codes: dict, scale_bits: int, d: int = D) -> np.ndarray:
     """One INT4 row: codes {element: code} (others 8, i.e. weight 0) and one scale per group."""
     c = np.full(d, 8, np.uint8)
     for i, v in codes.items():
         c[i] = v
-    packed = (c[0::2] | (c[1::2] << 4)).astype(np.uint8)
     scales = np.full(d // 32, scale_bits, np.uint16).astype("<u2").view(np.uint8)
-    return np.concatenate([packed, scales])
+    return np.concatenate([_pack(c), scales])
 
 
 def _bf16(v):
@@ -82,9 +115,7 @@ def test_int4_scale_decoding_matches_numpy_float16(oracle_mod, bits):
 
 def _numpy_dequant(q: np.ndarray, d: int) -> np.ndarray:
     """Independent decoding with numpy: nibbles, float16 view, broadcast per group."""
-    codes = np.empty((q.shape[0], d), np.int64)
-    codes[:, 0::2] = q[:, : d // 2] & 0x0F
-    codes[:, 1::2] = q[:, : d // 2] >> 4
+    codes = _unpack(q, d)
     scales = np.ascontiguousarray(q[:, d // 2:]).view("<f2").astype(np.float64)
     return np.repeat(scales, 32, axis=1) * (codes - 8)
 
@@ -119,11 +150,8 @@ def test_quantizer_round_trip_bound():
 
 
 def _planted(q_rows, d, mistake):
-    codes = np.empty((q_rows.shape[0], d), np.int64)
-    lo, hi = q_rows[:, : d // 2] & 0x0F, q_rows[:, : d // 2] >> 4
-    if mistake == "swapped_nibbles":
-        lo, hi = hi, lo
-    codes[:, 0::2], codes[:, 1::2] = lo, hi
+    codes = _unpack(q_rows, d, halves=(1, 0) if mistake == "swapped_halves" else (0, 1),
+                    sequential=mistake == "sequential")
     sc = np.ascontiguousarray(q_rows[:, d // 2:])
     scales = sc.view(">f2" if mistake == "big_endian_scale" else "<f2").astype(np.float64)
     per = np.repeat(scales, 32, axis=1)
@@ -133,7 +161,8 @@ def _planted(q_rows, d, mistake):
     return per * (codes - off)
 
 
-@pytest.mark.parametrize("mistake", ["swapped_nibbles", "offset_7", "big_endian_scale", "shifted_group"])
+@pytest.mark.parametrize("mistake", ["swapped_halves", "sequential", "offset_7", "big_endian_scale",
+                                     "shifted_group"])
 def test_int4_pins_reject_planted_mistakes(mistake):
     x, wg, wu, wd, y = _handworked()
     # the hand-worked case with a second group, so a shifted group is visible
