@@ -47,7 +47,7 @@ constexpr int kWindow = 8;     // chunks in flight per CTA
 constexpr int kLookahead = 3;  // gate chunks issued ahead of their up rows (< kWindow)
 constexpr int kMaxSlots = 32;
 constexpr int kRingBytes = 128 * 1024;  // ring budget: leaves room for down-projection CTAs
-constexpr int kSmemMargin = 8192;       // static shared memory headroom
+constexpr int kSmemMargin = 12288;      // static shared memory headroom
 
 enum : int { kTaskGate = 0, kTaskUp = 1, kTaskEnd = 2 };
 
@@ -87,11 +87,13 @@ struct GateUpShared {
     uint64_t full[kMaxSlots];
     uint64_t empty[kMaxSlots];
     uint64_t gate_ready[kWindow];
-    uint64_t chunk_free[kWindow];
+    // chunk states: kWindow, or two per consumer warp in the INT4 kernel
+    uint64_t chunk_free[NT <= kAccMaxTokens ? 2 * kWindow : kWindow];
     uint64_t never;  // nothing arrives here (FfnLaunch::test_stall)
     int mma_ok;      // tensor-core consumers: every wait so far succeeded
     Task task[kMaxSlots];
-    ChunkState<NT> cs[kWindow];
+    ChunkState<NT> cs[NT <= kAccMaxTokens ? 2 * kWindow : kWindow];
+    int next_chunk;  // INT4 kernel: next local chunk to claim
     ExpertSets es;
     float red[kMaxConsumers];
 };
@@ -341,8 +343,10 @@ __device__ __forceinline__ void partial_blocks(const FfnLaunch& a, GateUpShared<
         }
 }
 
-// INT4 rows: lane l of a warp covers 16 columns (8 code bytes, half a group,
-// one scale) of a 512-column block, for U rows at a time.
+// INT4 rows: in a 512-column block, lanes 2q and 2q+1 share group q (32
+// columns, 16 code bytes, one scale); lane parity p reads code words 2p and
+// 2p+1, which hold the group's columns 8s + 4p + {0..3} (s = 0..3). Each lane
+// so covers 16 columns, for U rows at a time.
 __device__ __forceinline__ uint2 ld_nc_u2(const void* p) {
     uint2 v;
     asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(p));
@@ -361,14 +365,17 @@ __device__ __forceinline__ void partial_blocks_q4(const FfnLaunch& a, GateUpShar
     constexpr int U = 8;
     const int d = a.d;
     const int n_slots = a.route ? a.batch : a.nt;
-    const int col = blk * 512 + lane * 16;
-    const bool valid = col < d;
+    const int grp = blk * 16 + lane / 2;
+    const int p = lane % 2;
+    const int col0 = grp * 32 + 4 * p;  // columns col0 + 8s + {0..3}
+    const bool valid = grp * 32 < d;
+    // acc[t][4s + c] is column col0 + 8s + c
     float acc[AT][16];
 #pragma unroll
     for (int t = 0; t < AT; ++t)
 #pragma unroll
         for (int v = 0; v < 16; ++v)
-            acc[t][v] = (accumulate && valid && t < n_slots) ? pbase[(size_t)t * d + col + v] : 0.0f;
+            acc[t][v] = (accumulate && valid && t < n_slots) ? pbase[(size_t)t * d + col0 + 8 * (v / 4) + v % 4] : 0.0f;
     for (int g = 0; g < n; g += U) {
         uint2 cw[U];
         float sc[U];
@@ -378,8 +385,8 @@ __device__ __forceinline__ void partial_blocks_q4(const FfnLaunch& a, GateUpShar
             cw[u] = make_uint2(0x88888888u, 0x88888888u);  // codes of weight 0
             sc[u] = 0.0f;
             if (row != nullptr && valid) {
-                cw[u] = ld_nc_u2(row + col / 2);
-                sc[u] = ld_nc_half(row + d / 2 + (col / 32) * 2);
+                cw[u] = ld_nc_u2(row + grp * 16 + 8 * p);
+                sc[u] = ld_nc_half(row + d / 2 + grp * 2);
             }
         }
 #pragma unroll
@@ -390,8 +397,11 @@ __device__ __forceinline__ void partial_blocks_q4(const FfnLaunch& a, GateUpShar
                 for (int t = 0; t < AT; ++t) c[t] = sh.pd.cs[g + u][t] * sc[u];
 #pragma unroll
                 for (int v = 0; v < 16; ++v) {
-                    const uint32_t word = v < 8 ? cw[u].x : cw[u].y;
-                    const float q = (float)((int)((word >> (4 * (v & 7))) & 15u) - 8);
+                    // column 8s + 2tw + h of the lane's pair: word tw, nibble s + 4h
+                    const int s4 = v / 4, tw = (v % 4) / 2, h = v % 2;
+                    const uint32_t word = tw ? cw[u].y : cw[u].x;
+                    // 2^23 + code as a float, minus 2^23 + 8: code - 8, exact
+                    const float q = __uint_as_float(0x4B000000u | ((word >> (4 * s4 + 16 * h)) & 15u)) - 8388616.0f;
 #pragma unroll
                     for (int t = 0; t < AT; ++t)
                         if (t < n_slots) acc[t][v] = fmaf(c[t], q, acc[t][v]);
@@ -403,9 +413,10 @@ __device__ __forceinline__ void partial_blocks_q4(const FfnLaunch& a, GateUpShar
 #pragma unroll
         for (int t = 0; t < AT; ++t)
             if (t < n_slots) {
-                float4* o = reinterpret_cast<float4*>(pbase + (size_t)t * d + col);
 #pragma unroll
-                for (int v = 0; v < 16; v += 4) o[v / 4] = make_float4(acc[t][v], acc[t][v + 1], acc[t][v + 2], acc[t][v + 3]);
+                for (int s4 = 0; s4 < 4; ++s4)
+                    *reinterpret_cast<float4*>(pbase + (size_t)t * d + col0 + 8 * s4) =
+                        make_float4(acc[t][4 * s4], acc[t][4 * s4 + 1], acc[t][4 * s4 + 2], acc[t][4 * s4 + 3]);
             }
     }
 }
@@ -803,7 +814,6 @@ struct MmaCfg {
     int lookahead;  // gate groups issued ahead of their chunk's up group
     int end_tasks;  // end groups to emit: 1 (all consumers read each group) or one per consumer
 };
-constexpr int kMmaMaxGroups = 8;
 
 // The producer of the tensor-core variant: groups in task order (gate rows of
 // chunk c, then the up rows of chunk c-1), one expect-tx barrier per group.
@@ -909,17 +919,8 @@ __device__ void produce_mma(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
 }
 
 // The consumers of the tensor-core variant (C warps, all on every group).
-// B fragment pair of two INT4 codes (low nibble = the lower k): bf16x2 of
-// (code - 8), exact. 0x4300 is 128.0 in bf16, whose last mantissa bit is 1.0,
-// so OR-ing a code into it gives 128 + code; subtracting 136 leaves code - 8.
-__device__ __forceinline__ uint32_t q4_pair(uint32_t byte) {
-    const uint32_t v = 0x43004300u | (byte & 0x0Fu) | ((byte & 0xF0u) << 12);
-    __nv_bfloat162 p = *reinterpret_cast<const __nv_bfloat162*>(&v);
-    p = __hsub2(p, __floats2bfloat162_rn(136.0f, 136.0f));
-    return *reinterpret_cast<const uint32_t*>(&p);
-}
 
-template <int NT, bool Q4>
+template <int NT>
 __device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsigned char* ring,
                             const unsigned char* xb, float* red, const MmaCfg& mc, int cidx, int lane) {
     constexpr int C = GateUpWarps<NT>::C;
@@ -955,7 +956,7 @@ __device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsi
         const Task tk = sh.task[g];
         if (tk.kind == kTaskEnd) return;
         float acc0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, acc1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-        if constexpr (!Q4) {
+        {
             const uint32_t w_addr = smem_u32(ring) + (g * kChunk + lane % 8) * mc.w_stride + (lane / 8) * 16;
             for (int ks = ks0; ks < ks0 + per; ks += 2) {
                 uint32_t a0, a2, a0n, a2n, b0, b1, b0n, b1n;
@@ -963,29 +964,6 @@ __device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsi
                 ldsm_x4(w_addr + ks * 32, b0, b1, b0n, b1n);
                 mma_bf16_16816(acc0, a0, a2, b0, b1);
                 mma_bf16_16816(acc1, a0n, a2n, b0n, b1n);
-            }
-        } else {
-            // INT4 rows: a K-step pair is one group of 32 codes (16 bytes) and
-            // one binary16 scale per row. Lane (row lane/4, pair lane%4) takes
-            // codes 2t, 2t+1 / 2t+8, 2t+9 of each K-step as its B fragment;
-            // the group's MMA sum is scaled per output column (rows 2t, 2t+1).
-            const int t = lane % 4;
-            const unsigned char* wrow = ring + ((size_t)g * kChunk + lane / 4) * mc.w_stride;
-            const unsigned char* s0row = ring + ((size_t)g * kChunk + 2 * t) * mc.w_stride + a.d / 2;
-            const unsigned char* s1row = s0row + mc.w_stride;
-            for (int ks = ks0; ks < ks0 + per; ks += 2) {
-                uint32_t a0, a2, a0n, a2n;
-                ldsm_x4(x_addr + ks * 32, a0, a2, a0n, a2n);
-                const uint4 cw = lds128(wrow + (size_t)ks * 8);
-                const int sh8 = 8 * t;
-                float dg[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-                mma_bf16_16816(dg, a0, a2, q4_pair((cw.x >> sh8) & 0xFFu), q4_pair((cw.y >> sh8) & 0xFFu));
-                mma_bf16_16816(dg, a0n, a2n, q4_pair((cw.z >> sh8) & 0xFFu), q4_pair((cw.w >> sh8) & 0xFFu));
-                const int grp32 = ks / 2;
-                const float sc0 = __half2float(*reinterpret_cast<const __half*>(s0row + grp32 * 2));
-                const float sc1 = __half2float(*reinterpret_cast<const __half*>(s1row + grp32 * 2));
-                acc0[0] = fmaf(sc0, dg[0], acc0[0]);
-                acc0[1] = fmaf(sc1, dg[1], acc0[1]);
             }
         }
         __syncwarp();
@@ -1043,7 +1021,7 @@ __device__ void consume_mma(const FfnLaunch& a, GateUpShared<NT>& sh, const unsi
     }
 }
 
-template <int NT, bool Q4>
+template <int NT>
 __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_mma(const FfnLaunch a, const MmaCfg mc) {
     using T = __nv_bfloat16;  // activations (and bf16 weights)
     constexpr int C = GateUpWarps<NT>::C;
@@ -1062,9 +1040,6 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_mma(con
             mbar_init(&sh.empty[g], C);
         }
         mbar_init(&sh.never, 1);
-        if constexpr (NT <= kAccMaxTokens) {
-            for (int q = 0; q < kMaxLocal; ++q) sh.pd.ub[q] = 0;
-        }
         for (int w = 0; w < kWindow; ++w) {
             mbar_init(&sh.gate_ready[w], 1);
             mbar_init(&sh.chunk_free[w], 1);
@@ -1113,29 +1088,20 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_mma(con
         }
     }
     named_bar_sync(1, cthreads);
-    consume_mma<NT, Q4>(a, sh, ring, xb, red, mc, warp - 1, lane);
-    if constexpr (NT <= kAccMaxTokens) {
-        // every chunk is finalized once all consumers are here
-        named_bar_sync(1, cthreads);
-        down_partial<T, NT, Q4>(a, sh, i0, i1, n_chunks, warp - 1, lane);
-    }
+    consume_mma<NT>(a, sh, ring, xb, red, mc, warp - 1, lane);
 }
 
 // Shared memory of the tensor-core variant: activations, the cross-warp
-// sums of every group in flight, and the ring. bf16 rows keep kMmaGroups
-// groups in flight; INT4 rows, 3.6x smaller, as many as fit (up to
-// kMmaMaxGroups) so about as many bytes are in flight.
-static size_t mma_smem(int wdtype, int d, int avail, MmaCfg* mc) {
-    const int row_bytes = wdtype == 2 ? d / 2 + d / 16 : d * 2;
+// sums of every group in flight, and the ring of kMmaGroups bf16 groups.
+static size_t mma_smem(int d, MmaCfg* mc) {
+    const int row_bytes = d * 2;
     mc->x_stride = d * 2 + kMmaRowPad;
     mc->w_stride = row_bytes + kMmaRowPad;
     auto bytes = [&](int g) {
         return (size_t)kChunk * mc->x_stride + (size_t)g * GateUpWarps<8>::C * 64 * sizeof(float) +
                (size_t)g * kChunk * mc->w_stride;
     };
-    int g = kMmaGroups;
-    if (wdtype == 2)
-        while (g < kMmaMaxGroups && bytes(g + 1) <= (size_t)avail) ++g;
+    const int g = kMmaGroups;
     mc->groups = g;
     mc->lookahead = 1;
     mc->end_tasks = 1;
@@ -1143,99 +1109,311 @@ static size_t mma_smem(int wdtype, int d, int avail, MmaCfg* mc) {
 }
 
 // ---------------------------------------------------------------------------
-// INT4 rows, passes of 1-2 tokens: each consumer warp takes whole groups (a
-// chunk's 8 gate rows, or its gate-active up rows) over the full K, so no
-// warp waits on another: INT4 rows are 3.6x smaller than bf16 rows, and the
-// shared-group design above would spend more time in its per-group barriers
-// than in the MMAs. Consumer warp c owns ring slot c (one group each).
+// INT4 rows, passes of 1-2 tokens. A subtask is up to kQ4Rows rows of one
+// chunk (its gate rows, or its gate-active up rows) over the full K,
+// computed by one consumer warp from one of its two ring slots.
+//
+// One m16n8k16 MMA covers the task's 4 rows over all four K-quarters: A row
+// g (g < 8) is task row g % 4 over quarter g / 4, A row g + 8 the same row
+// over quarter 3 - g / 4; B column n is token n / 4 over quarter (n even:
+// (n / 2) % 2, n odd: 2 + (n / 2) % 2). Each lane then holds exactly one
+// product of matching quarters, D[g][2t] when g / 4 == t % 2 and
+// D[g + 8][2t + 1] otherwise, and the four quarters of a (row, token) sit in
+// lanes {l, l ^ 1, l ^ 16, l ^ 17}. Odd quarters walk each pair of groups in
+// swapped order, which keeps the lanes' shared-memory words in distinct banks.
 // ---------------------------------------------------------------------------
-constexpr int kQ4Lookahead = 5;  // gate groups ahead of their up group (< kWindow)
+constexpr int kQ4Rows = 4;          // rows per subtask
+constexpr int kQ4SlotsPerWarp = 2;  // ring slots per consumer warp
+constexpr int kQ4QuarterPad = 16;   // bytes after each K-quarter of an activation row
+
+// bf16x2 A-fragment register of two INT4 codes held at bits 0-3 and 16-19
+// of v: (code_lo - 8, code_hi - 8), exact. 0x4300 is 128.0 in bf16, whose
+// last mantissa bit is worth 1.0, so OR-ing a code into it gives 128 + code;
+// subtracting 136 leaves code - 8.
+__device__ __forceinline__ uint32_t q4_frag(uint32_t v) {
+    const uint32_t b = (v & 0x000F000Fu) | 0x43004300u;
+    __nv_bfloat162 p = *reinterpret_cast<const __nv_bfloat162*>(&b);
+    p = __hsub2(p, __floats2bfloat162_rn(136.0f, 136.0f));
+    return *reinterpret_cast<const uint32_t*>(&p);
+}
+__device__ __forceinline__ uint32_t lds32(const void* p) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(smem_u32(p)));
+    return v;
+}
+// d += A * B for one m16n8k16 step with all 16 A rows.
+__device__ __forceinline__ void mma_bf16_16816_a4(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                                  uint32_t b0, uint32_t b1) {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Each consumer warp owns whole chunks, claimed in order from a counter
+// shared by the CTA's warps, and works through them in subtasks of up to
+// kQ4Rows rows: the chunk's gate rows, then its gate-active up rows. The
+// warp copies the rows of its next subtask (16-byte cp.async per lane, into
+// the other of its two slots) before it computes the current one. The
+// order G_k.0, G_k.1, G_k'.0, U_k, G_k'.1, G_k''.0, U_k', ... (the up rows
+// of a finished gate first, else pending gate rows, else a new chunk) keeps
+// one subtask between a chunk's last gate rows and its up rows, so their
+// copies are in flight while the warp computes; a warp holds at most two
+// chunks. No warp waits on another until the down projection.
+struct Q4Sub {
+    int kind;       // kTaskGate, kTaskUp, or kTaskEnd (nothing left)
+    int ci;         // the warp's chunk (0 or 1)
+    unsigned rows;  // chunk rows of the subtask (at most kQ4Rows)
+};
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
 
 template <int NT>
-__device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, const unsigned char* ring,
-                            const unsigned char* xb, const MmaCfg& mc, int cidx, int lane) {
-    constexpr int C = GateUpWarps<NT>::C;
+__device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char* ring, const unsigned char* xb,
+                            const MmaCfg& mc, int i0, int i1, int n_chunks, int cidx, int lane) {
     const int d = a.d;
-    const int t = lane % 4;
-    const uint32_t x_addr = smem_u32(xb) + (lane % 8) * mc.x_stride + (lane / 8) * 16;
-    const unsigned slot = (unsigned)cidx;  // groups == C: this warp's only slot
-    unsigned phase = 0;
+    const int nq = d / 128;  // 32-element groups per K-quarter
+    const int g = lane / 4, t = lane % 4;
+    const int wr = g % 4;                  // task row of this lane's A rows
+    const int qa = g / 4, qb = 3 - g / 4;  // their K-quarters
+    const bool use_d0 = qa == (t & 1);     // which D element holds this lane's product
+    const int qu = use_d0 ? qa : qb;       // the quarter of that product
+    // A words: word t of each group of the lane's two quarters; odd quarters
+    // take the pair (G, G + 1) in the order (G + 1, G)
+    const int a_off0 = (qa & 1) * 16, a_off1 = 16 - a_off0;
+    const int b_off0 = (qb & 1) * 16, b_off1 = 16 - b_off0;
+    // B: this lane addresses column n = lane % 8 for ldmatrix; with one
+    // token, columns 4-7 repeat token 0 (same addresses, no bank conflict)
+    // and their products are not used
+    const int n = lane % 8;
+    const int n_tok = NT > 1 ? n / 4 : 0;
+    const int n_q = (n & 1) ? 2 + ((n >> 1) & 1) : ((n >> 1) & 1);
+    const uint32_t x_col = smem_u32(xb) + n_tok * mc.x_stride + n_q * (d / 2 + kQ4QuarterPad) + (lane / 8) * 16;
+    const uint32_t x_step = 64u;
+    const uint32_t x_off0 = (n_q & 1) ? x_step : 0u, x_off1 = x_step - x_off0;
+    const unsigned row_bytes = (unsigned)a.row_bytes;
+    const int row_chunks = (int)(row_bytes / 16);
+    const int n_local = i1 - i0;
     if (a.test_stall && cidx == 0) {
-        // the failure-detection test: a wait that can only run out
-        if (!warp_wait(&sh.never, 0u, lane, a.status)) return;
+        // the failure-detection test: a wait that can only run out (the
+        // other warps take every chunk)
+        warp_wait(&sh.never, 0u, lane, a.status);
+        return;
     }
-    for (;;) {
-        if (!warp_wait(&sh.full[slot], phase, lane, a.status)) return;
-        phase ^= 1u;
-        const Task tk = sh.task[slot];
-        if (tk.kind == kTaskEnd) return;
-        const unsigned char* base = ring + (size_t)slot * kChunk * mc.w_stride;
-        const unsigned char* wrow = base + (size_t)(lane / 4) * mc.w_stride;
-        const unsigned char* s0row = base + (size_t)(2 * t) * mc.w_stride + d / 2;
-        const unsigned char* s1row = s0row + mc.w_stride;
-        float v0a = 0.0f, v1a = 0.0f, v0b = 0.0f, v1b = 0.0f;  // two chains (even / odd groups)
-        const int sh8 = 8 * t;
-        for (int gq = 0; gq < d / 32; gq += 2) {
+
+    // the warp's two chunks: chunk state 2 * cidx + ci
+    int st[2] = {0, 0};           // 0 free, 1 gate rows pending, 2 up rows pending
+    unsigned left[2] = {0u, 0u};  // rows not yet handed to a subtask (gate, then up)
+    int gate_subs[2] = {0, 0};    // gate subtasks not yet computed
+    int up_rows[2] = {0, 0};      // up rows not yet computed
+    int older = 0;                // the chunk claimed first
+    bool more = true;             // chunks may remain to claim
+
+    auto take = [&](unsigned& m) {
+        unsigned sub = 0u;
+        for (int i = 0; i < kQ4Rows && m != 0u; ++i) {
+            sub |= m & (0u - m);
+            m &= m - 1u;
+        }
+        return sub;
+    };
+    // claim the next chunk with rows into state ci: its rows, expert and local index
+    auto claim = [&](int ci) -> bool {
+        while (more) {
+            int c = 0;
+            if (lane == 0) c = atomicAdd(&sh.next_chunk, 1);
+            c = __shfl_sync(0xffffffffu, c, 0);
+            if (c >= n_local) {
+                more = false;
+                return false;
+            }
+            const int item = i0 + c;
+            const int ea = item / n_chunks;
+            const int chunk = item - ea * n_chunks;
+            const int e = sh.es.act[ea];
+            volatile ChunkState<NT>& s = sh.cs[2 * cidx + ci];
+            int j = -1;
+            const int p = chunk * kChunk + lane;
+            if (lane < kChunk && p < a.n_rows) {
+                if (a.rows != nullptr) {
+                    const int jj = a.rows[p];
+                    if ((unsigned)jj < (unsigned)a.m && (p == 0 || a.rows[p - 1] < jj))
+                        j = jj;
+                    else
+                        atomicOr(a.status, kStatusBadIndex);
+                } else {
+                    j = p;
+                }
+            }
+            if (lane < kChunk) s.jr[lane] = j;
+            const unsigned mask = __ballot_sync(0xffffffffu, j >= 0);
+            if (lane == 0) {
+                s.e = e;
+                s.chunk = chunk;
+                s.q = c;
+                s.n_gate = __popc(mask);
+                s.gate_cnt = 0;
+                s.up_cnt = 0;
+                s.gmask = 0u;
+            }
+            __syncwarp();
+            if (mask == 0u) {
+                // no rows here: nothing active
+                const int ntok = sh.es.ntok[e];
+                if (lane < ntok) {
+                    const size_t tb = (size_t)(a.bits_tok_base + lane) * a.nbytes;
+                    a.gbits[(size_t)e * a.bits_expert_stride + chunk + tb] = 0;
+                    a.bbits[(size_t)e * a.bits_expert_stride + chunk + tb] = 0;
+                }
+                if (lane == 0) {
+                    a.ubits[(size_t)e * a.nbytes + chunk] = 0;
+                    a.ugbits[(size_t)e * a.nbytes + chunk] = 0;
+                    if (c < kMaxLocal) sh.pd.ub[c] = 0;
+                }
+                continue;
+            }
+            st[ci] = 1;
+            left[ci] = mask;
+            gate_subs[ci] = (__popc(mask) + kQ4Rows - 1) / kQ4Rows;
+            older = st[ci ^ 1] != 0 ? (ci ^ 1) : ci;
+            return true;
+        }
+        return false;
+    };
+    // the next subtask: the up rows of a finished gate (older chunk first),
+    // else pending gate rows, else a newly claimed chunk's first gate rows
+    auto pick = [&]() -> Q4Sub {
+        for (int k = 0; k < 2; ++k) {
+            const int ci = k == 0 ? older : older ^ 1;
+            if (st[ci] == 2 && left[ci] != 0u) return Q4Sub{kTaskUp, ci, take(left[ci])};
+        }
+        for (int k = 0; k < 2; ++k) {
+            const int ci = k == 0 ? older : older ^ 1;
+            if (st[ci] == 1 && left[ci] != 0u) return Q4Sub{kTaskGate, ci, take(left[ci])};
+        }
+        for (int ci = 0; ci < 2; ++ci)
+            if (st[ci] == 0 && claim(ci)) return Q4Sub{kTaskGate, ci, take(left[ci])};
+        return Q4Sub{kTaskEnd, 0, 0u};
+    };
+    // copy a subtask's rows into this warp's slot `slot` (one commit group)
+    auto issue = [&](const Q4Sub& sb, int slot) {
+        volatile ChunkState<NT>& s = sh.cs[2 * cidx + sb.ci];
+        const int e = s.e;
+        const unsigned char* w = static_cast<const unsigned char*>(sb.kind == kTaskGate ? a.ex[e].wg : a.ex[e].wu);
+        unsigned char* dst = ring + (size_t)(2 * cidx + slot) * kQ4Rows * mc.w_stride;
+        int i = 0;
+        for (unsigned m = sb.rows; m; m &= m - 1u, ++i) {
+            const int j = s.jr[__ffs(m) - 1];
+            const unsigned char* src = w + (size_t)j * row_bytes;
+            unsigned char* drow = dst + (size_t)i * mc.w_stride;
+            for (int c = lane; c < row_chunks; c += kWarp) cp_async16(drow + 16 * c, src + 16 * c);
+        }
+        cp_async_commit();
+    };
+
+    Q4Sub cur = pick();
+    int slot = 0;
+    if (cur.kind != kTaskEnd) issue(cur, slot);
+    while (cur.kind != kTaskEnd) {
+        const Q4Sub nxt = pick();
+        if (nxt.kind != kTaskEnd) {
+            issue(nxt, slot ^ 1);
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        __syncwarp();  // every lane's copies of the current subtask have landed
+        const unsigned char* row = ring + ((size_t)(2 * cidx + slot) * kQ4Rows + wr) * mc.w_stride;
+        const unsigned char* wa = row + qa * (d / 8) + 4 * t;
+        const unsigned char* wb = row + qb * (d / 8) + 4 * t;
+        const unsigned char* sp = row + d / 2 + qu * nq * 2;  // binary16 scales of quarter qu
+        float v0 = 0.0f, v1 = 0.0f;
+#pragma unroll 2
+        for (int G = 0; G < nq; G += 2) {
+            const float2 sc = __half22float2(*reinterpret_cast<const __half2*>(sp + G * 2));
+            const float s0 = (qu & 1) ? sc.y : sc.x;
+            const float s1 = (qu & 1) ? sc.x : sc.y;
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-                const int ks = 2 * (gq + h);
-                uint32_t a0, a2, a0n, a2n;
-                ldsm_x4(x_addr + ks * 32, a0, a2, a0n, a2n);
-                const uint4 cw = lds128(wrow + (size_t)ks * 8);
+                uint32_t b0, b1, b0n, b1n;
+                ldsm_x4(x_col + G * x_step + (h ? x_off1 : x_off0), b0, b1, b0n, b1n);
+                const uint32_t ca = lds32(wa + G * 16 + (h ? a_off1 : a_off0));
+                const uint32_t cb = lds32(wb + G * 16 + (h ? b_off1 : b_off0));
                 float dg[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-                mma_bf16_16816(dg, a0, a2, q4_pair((cw.x >> sh8) & 0xFFu), q4_pair((cw.y >> sh8) & 0xFFu));
-                mma_bf16_16816(dg, a0n, a2n, q4_pair((cw.z >> sh8) & 0xFFu), q4_pair((cw.w >> sh8) & 0xFFu));
-                const float sc0 = __half2float(*reinterpret_cast<const __half*>(s0row + (gq + h) * 2));
-                const float sc1 = __half2float(*reinterpret_cast<const __half*>(s1row + (gq + h) * 2));
-                if (h == 0) {
-                    v0a = fmaf(sc0, dg[0], v0a);
-                    v1a = fmaf(sc1, dg[1], v1a);
-                } else {
-                    v0b = fmaf(sc0, dg[0], v0b);
-                    v1b = fmaf(sc1, dg[1], v1b);
-                }
+                // element 8s + 2t + {0, 1} of a group is nibble s (+4) of word t
+                mma_bf16_16816_a4(dg, q4_frag(ca), q4_frag(cb), q4_frag(ca >> 4), q4_frag(cb >> 4), b0, b1);
+                mma_bf16_16816_a4(dg, q4_frag(ca >> 8), q4_frag(cb >> 8), q4_frag(ca >> 12), q4_frag(cb >> 12), b0n,
+                                  b1n);
+                const float pv = use_d0 ? dg[0] : dg[3];
+                if (h == 0)
+                    v0 = fmaf(s0, pv, v0);
+                else
+                    v1 = fmaf(s1, pv, v1);
             }
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sh.empty[slot]);
-        // D row = token lane/4, columns = rows 2t, 2t+1 of the group
-        volatile ChunkState<NT>& s = sh.cs[tk.cw];
+        // the four K-quarters of (row wr, token t / 2), in the same order in every lane
+        float v = v0 + v1;
+        v += __shfl_xor_sync(0xffffffffu, v, 1);
+        v += __shfl_xor_sync(0xffffffffu, v, 16);
+        const int ci = cur.ci;
+        const int cs_i = 2 * cidx + ci;
+        volatile ChunkState<NT>& s = sh.cs[cs_i];
         const int e = s.e;
         const int ntok = sh.es.ntok[e];
-        const int tok = lane / 4;
-        const float v[2] = {v0a + v0b, v1a + v1b};
+        if (g < kQ4Rows && (t & 1) == 0 && wr < __popc(cur.rows)) {
+            const int r = __fns(cur.rows, 0, wr + 1);  // chunk row of task row wr
+            const int tok = t / 2;
 #pragma unroll
-        for (int q = 0; q < 2; ++q) {
-            const int r = 2 * t + q;
-            if ((tk.r >> r) & 1) {
-#pragma unroll
-                for (int k = 0; k < NT; ++k) {
-                    const int tk_x = a.route ? sh.es.tok[e][k] : k;
-                    if (k < ntok && tk_x == tok) {
-                        if (tk.kind == kTaskGate)
-                            s.g[r][k] = v[q];
-                        else
-                            s.u[r][k] = v[q];
-                    }
+            for (int k = 0; k < NT; ++k) {
+                const int tk_x = a.route ? sh.es.tok[e][k] : k;
+                if (k < ntok && tk_x == tok) {
+                    if (cur.kind == kTaskGate)
+                        s.g[r][k] = v;
+                    else
+                        s.u[r][k] = v;
                 }
             }
         }
         __syncwarp();
-        __threadfence_block();
-        if (tk.kind == kTaskGate) {
-            bool ga = false;
-            if (lane < kChunk && s.jr[lane] >= 0) {
+        bool done = false;
+        if (cur.kind == kTaskGate) {
+            if (--gate_subs[ci] == 0) {
+                // every gate row of the chunk is in: which rows need their W_up row?
+                bool ga = false;
+                if (lane < kChunk && s.jr[lane] >= 0) {
 #pragma unroll
-                for (int k = 0; k < NT; ++k) ga |= (k < ntok) && (s.g[lane][k] > 0.0f);
+                    for (int k = 0; k < NT; ++k) ga |= (k < ntok) && (s.g[lane][k] > 0.0f);
+                }
+                const unsigned gm = __ballot_sync(0xffffffffu, ga);
+                if (lane == 0) s.gmask = gm;
+                __syncwarp();
+                st[ci] = 2;
+                left[ci] = gm;
+                up_rows[ci] = __popc(gm);
+                done = gm == 0u;
             }
-            const unsigned gm = __ballot_sync(0xffffffffu, ga);
-            if (lane == 0) s.gmask = gm;
-            __syncwarp();
-            __threadfence_block();
-            if (gm == 0u) finalize_chunk<NT>(a, sh, tk.cw, lane);
-            if (lane == 0) mbar_arrive(&sh.gate_ready[tk.cw]);
         } else {
-            finalize_chunk<NT>(a, sh, tk.cw, lane);
+            up_rows[ci] -= __popc(cur.rows);
+            done = up_rows[ci] == 0;
+        }
+        if (done) {
+            finalize_chunk<NT>(a, sh, cs_i, lane);
+            st[ci] = 0;
+            older = ci ^ 1;
+        }
+        cur = nxt;
+        slot ^= 1;
+        if (cur.kind == kTaskEnd) {
+            // up rows of a chunk whose gate finished just now may still be due
+            cur = pick();
+            if (cur.kind != kTaskEnd) issue(cur, slot);
         }
     }
 }
@@ -1246,23 +1424,19 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
     constexpr int C = GateUpWarps<NT>::C;
     __shared__ GateUpShared<NT> sh;
     extern __shared__ __align__(128) unsigned char dyn[];
-    unsigned char* xb = dyn;                                     // [8][x_stride] bf16 activations
-    unsigned char* ring = dyn + (size_t)kChunk * mc.x_stride;    // [C][8][w_stride]
+    // [NT][4 quarters][d/4 bf16 + pad] activations
+    unsigned char* xb = dyn;
+    const size_t x_bytes = ((size_t)kAccMaxTokens * mc.x_stride + 127) / 128 * 128;
+    unsigned char* ring = dyn + x_bytes;  // [C][2 slots][kQ4Rows][w_stride]
     const int n_x = a.route ? a.batch : a.nt;
 
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     if (threadIdx.x == 0) {
-        for (int g = 0; g < mc.groups; ++g) {
-            mbar_init(&sh.full[g], 1);
-            mbar_init(&sh.empty[g], 1);
-        }
         mbar_init(&sh.never, 1);
         for (int q = 0; q < kMaxLocal; ++q) sh.pd.ub[q] = 0;
-        for (int w = 0; w < kWindow; ++w) {
-            mbar_init(&sh.gate_ready[w], 1);
-            mbar_init(&sh.chunk_free[w], 1);
-        }
+        for (int w = 0; w < 2 * kWindow; ++w) mbar_init(&sh.chunk_free[w], 1);
+        sh.next_chunk = 0;
         mbar_fence_init();
     }
     const bool early = a.rows == nullptr && a.route == nullptr;
@@ -1275,18 +1449,17 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
     const int i0 = (int)((long long)n_items * blockIdx.x / gridDim.x);
     const int i1 = (int)((long long)n_items * (blockIdx.x + 1) / gridDim.x);
 
-    if (warp == 0) {
-        if (lane == 0) produce_mma<NT>(a, sh, ring, mc, i0, i1, n_chunks);
-        return;
-    }
+    if (warp == 0) return;  // the consumer warps copy their own rows
     if (early) pdl_wait();
     const int ctid = threadIdx.x - kWarp;
     const int cthreads = C * kWarp;
     const int x_tok0 = a.route ? 0 : a.tok0;
-    for (int t = 0; t < kChunk; ++t) {
+    const int dq = a.d / 4;
+    auto xpos = [&](int i) { return (i / dq) * (dq + kQ4QuarterPad / 2) + i % dq; };  // bf16 index in a row
+    for (int t = 0; t < NT; ++t) {
         __nv_bfloat16* xrow = reinterpret_cast<__nv_bfloat16*>(xb + (size_t)t * mc.x_stride);
         if (t >= n_x) {
-            for (int i = ctid; i < a.d; i += cthreads) xrow[i] = __float2bfloat16_rn(0.0f);
+            for (int i = ctid; i < a.d; i += cthreads) xrow[xpos(i)] = __float2bfloat16_rn(0.0f);
         } else if (a.norm_from_h) {
             const float* hr = a.h + (size_t)(x_tok0 + t) * a.d;
             float ss = 0.0f;
@@ -1298,27 +1471,37 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
             for (int w = 0; w < C; ++w) tot += sh.red[w];
             const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)a.d), 1e-5f));
             for (int i = ctid; i < a.d; i += cthreads)
-                xrow[i] = __float2bfloat16_rn((i == a.d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hr[i], rms)));
+                xrow[xpos(i)] =
+                    __float2bfloat16_rn((i == a.d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hr[i], rms)));
             named_bar_sync(1, cthreads);
         } else {
             const T* xr = static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d;
-            for (int i = ctid; i < a.d; i += cthreads) xrow[i] = xr[i];
+            for (int i = ctid; i < a.d; i += cthreads) xrow[xpos(i)] = xr[i];
         }
     }
     named_bar_sync(1, cthreads);
-    consume_q4w<NT>(a, sh, ring, xb, mc, warp - 1, lane);
+    consume_q4w<NT>(a, sh, ring, xb, mc, i0, i1, n_chunks, warp - 1, lane);
     // every chunk is finalized once all consumers are here
     named_bar_sync(1, cthreads);
     down_partial<T, NT, true>(a, sh, i0, i1, n_chunks, warp - 1, lane);
 }
 
-static size_t q4w_smem(int d, MmaCfg* mc) {
-    mc->x_stride = d * 2 + kMmaRowPad;
-    mc->w_stride = d / 2 + d / 16 + kMmaRowPad;
-    mc->groups = GateUpWarps<1>::C;
-    mc->lookahead = kQ4Lookahead;
-    mc->end_tasks = GateUpWarps<1>::C;
-    return (size_t)kChunk * mc->x_stride + (size_t)mc->groups * kChunk * mc->w_stride;
+// Shared memory of the INT4 kernel: activations (kAccMaxTokens rows of four
+// padded K-quarters), then the ring. A slot row's stride is
+// 32 bytes past a multiple of 128, which with the swapped order of odd
+// quarters puts the 32 lanes' code words in 32 banks.
+static size_t q4w_smem(int d, int avail, MmaCfg* mc) {
+    const int row_bytes = d / 2 + d / 16;
+    mc->x_stride = 4 * (d / 2 + kQ4QuarterPad);
+    mc->w_stride = row_bytes + ((32 - row_bytes % 128) % 128 + 128) % 128;
+    const size_t x_bytes = ((size_t)kAccMaxTokens * mc->x_stride + 127) / 128 * 128;
+    const int C = GateUpWarps<1>::C;
+    const size_t slot = (size_t)kQ4Rows * mc->w_stride;
+    mc->groups = C * kQ4SlotsPerWarp;
+    mc->lookahead = 0;
+    mc->end_tasks = 0;
+    (void)avail;
+    return x_bytes + (size_t)mc->groups * slot;
 }
 
 // ---------------------------------------------------------------------------
@@ -1368,10 +1551,10 @@ static cudaError_t launch_t(const FfnLaunch& a, int grid, cudaStream_t stream, b
     return cudaLaunchKernelEx(&lc, k_gate_up<T, NT>, a, cfg);
 }
 
-template <int NT, bool Q4>
+template <int NT>
 static cudaError_t launch_mma_t(const FfnLaunch& a, int grid, cudaStream_t stream, bool pdl) {
     MmaCfg mc;
-    const size_t smem = mma_smem(Q4 ? 2 : 1, a.d, g_optin - kSmemMargin, &mc);
+    const size_t smem = mma_smem(a.d, &mc);
     if (smem + kSmemMargin > (size_t)g_optin) return cudaErrorInvalidValue;
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(grid);
@@ -1383,13 +1566,13 @@ static cudaError_t launch_mma_t(const FfnLaunch& a, int grid, cudaStream_t strea
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = attr;
     lc.numAttrs = pdl ? 1 : 0;
-    return cudaLaunchKernelEx(&lc, k_gate_up_mma<NT, Q4>, a, mc);
+    return cudaLaunchKernelEx(&lc, k_gate_up_mma<NT>, a, mc);
 }
 
 template <int NT>
 static cudaError_t launch_q4w_t(const FfnLaunch& a, int grid, cudaStream_t stream, bool pdl) {
     MmaCfg mc;
-    const size_t smem = q4w_smem(a.d, &mc);
+    const size_t smem = q4w_smem(a.d, g_optin - kSmemMargin, &mc);
     if (smem + kSmemMargin > (size_t)g_optin) return cudaErrorInvalidValue;
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(grid);
@@ -1409,13 +1592,13 @@ constexpr int kMmaMinTokens = 4;  // narrowest bf16 pass that takes the tensor-c
 static bool use_mma(int wdtype, int d, int pass_tokens) {
     MmaCfg mc;
     return wdtype == 1 && pass_tokens >= kMmaMinTokens && d % kMmaDAlign == 0 &&
-           mma_smem(wdtype, d, g_optin - kSmemMargin, &mc) + kSmemMargin <= (size_t)g_optin;
+           mma_smem(d, &mc) + kSmemMargin <= (size_t)g_optin;
 }
 
 bool int4_supported(int d, int pass_tokens, int optin_smem) {
     MmaCfg mc;
     return d % kMmaDAlign == 0 && pass_tokens >= 1 && pass_tokens <= kAccMaxTokens &&
-           q4w_smem(d, &mc) + kSmemMargin <= (size_t)optin_smem;
+           q4w_smem(d, optin_smem - kSmemMargin, &mc) + kSmemMargin <= (size_t)optin_smem;
 }
 
 template <typename T, int NT>
@@ -1439,10 +1622,8 @@ cudaError_t prepare_gate_up(int optin_smem) {
     if (e == cudaSuccess) e = prepare_t<float, 4>(optin_smem);
     if (e == cudaSuccess) e = prepare_t<float, 8>(optin_smem);
     const int dyn = optin_smem - kSmemMargin;
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<4, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<8, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_q4w<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_q4w<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     return e;
@@ -1458,10 +1639,8 @@ cudaError_t launch_gate_up(const FfnLaunch& a, int wdtype, int pass_tokens, int 
         return cudaErrorInvalidValue;
     }
     if (use_mma(wdtype, a.d, pass_tokens)) {
-        if (pass_tokens == 1) return launch_mma_t<1, false>(a, grid, stream, pdl);
-        if (pass_tokens == 2) return launch_mma_t<2, false>(a, grid, stream, pdl);
-        if (pass_tokens == 4) return launch_mma_t<4, false>(a, grid, stream, pdl);
-        if (pass_tokens == 8) return launch_mma_t<8, false>(a, grid, stream, pdl);
+        if (pass_tokens == 4) return launch_mma_t<4>(a, grid, stream, pdl);
+        if (pass_tokens == 8) return launch_mma_t<8>(a, grid, stream, pdl);
     }
     if (wdtype == 1) {
         switch (pass_tokens) {
