@@ -47,7 +47,7 @@ constexpr int kWindow = 8;     // chunks in flight per CTA
 constexpr int kLookahead = 3;  // gate chunks issued ahead of their up rows (< kWindow)
 constexpr int kMaxSlots = 32;
 constexpr int kRingBytes = 128 * 1024;  // ring budget: leaves room for down-projection CTAs
-constexpr int kSmemMargin = 12288;      // static shared memory headroom
+constexpr int kSmemMargin = 8192;       // static shared memory headroom
 
 enum : int { kTaskGate = 0, kTaskUp = 1, kTaskEnd = 2 };
 
@@ -87,13 +87,13 @@ struct GateUpShared {
     uint64_t full[kMaxSlots];
     uint64_t empty[kMaxSlots];
     uint64_t gate_ready[kWindow];
-    // chunk states: kWindow, or two per consumer warp in the INT4 kernel
-    uint64_t chunk_free[NT <= kAccMaxTokens ? 2 * kWindow : kWindow];
+    uint64_t chunk_free[kWindow];
     uint64_t never;  // nothing arrives here (FfnLaunch::test_stall)
     int mma_ok;      // tensor-core consumers: every wait so far succeeded
     Task task[kMaxSlots];
-    ChunkState<NT> cs[NT <= kAccMaxTokens ? 2 * kWindow : kWindow];
-    int next_chunk;  // INT4 kernel: next local chunk to claim
+    ChunkState<NT> cs[kWindow];
+    int q4_ctr[4];                 // INT4 kernel: subtasks claimed per phase, up subtasks
+    unsigned q4_up[2 * kMaxLocal];  // INT4 kernel: up subtasks (chunk << 8 | rows)
     ExpertSets es;
     float red[kMaxConsumers];
 };
@@ -182,8 +182,7 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, unsigned parity, int la
 // Write a finished chunk's outputs (warp-wide) and free its window slot:
 // per-token gate/both bitmap bytes, union bytes, and c by batch slot.
 template <int NT>
-__device__ void finalize_chunk(const FfnLaunch& a, GateUpShared<NT>& sh, int cw, int lane) {
-    volatile ChunkState<NT>& s = sh.cs[cw];
+__device__ void finalize_chunk_s(const FfnLaunch& a, GateUpShared<NT>& sh, volatile ChunkState<NT>& s, int lane) {
     const int e = s.e;
     const int chunk = s.chunk;
     const int ntok = sh.es.ntok[e];
@@ -264,6 +263,10 @@ __device__ void finalize_chunk(const FfnLaunch& a, GateUpShared<NT>& sh, int cw,
         }
     }
     __syncwarp();
+}
+template <int NT>
+__device__ void finalize_chunk(const FfnLaunch& a, GateUpShared<NT>& sh, int cw, int lane) {
+    finalize_chunk_s<NT>(a, sh, sh.cs[cw], lane);
     __threadfence_block();
     if (lane == 0) mbar_arrive(&sh.chunk_free[cw]);
 }
@@ -1150,21 +1153,17 @@ __device__ __forceinline__ void mma_bf16_16816_a4(float (&d)[4], uint32_t a0, ui
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Each consumer warp owns whole chunks, claimed in order from a counter
-// shared by the CTA's warps, and works through them in subtasks of up to
-// kQ4Rows rows: the chunk's gate rows, then its gate-active up rows. The
-// warp copies the rows of its next subtask (16-byte cp.async per lane, into
-// the other of its two slots) before it computes the current one. The
-// order G_k.0, G_k.1, G_k'.0, U_k, G_k'.1, G_k''.0, U_k', ... (the up rows
-// of a finished gate first, else pending gate rows, else a new chunk) keeps
-// one subtask between a chunk's last gate rows and its up rows, so their
-// copies are in flight while the warp computes; a warp holds at most two
-// chunks. No warp waits on another until the down projection.
-struct Q4Sub {
-    int kind;       // kTaskGate, kTaskUp, or kTaskEnd (nothing left)
-    int ci;         // the warp's chunk (0 or 1)
-    unsigned rows;  // chunk rows of the subtask (at most kQ4Rows)
-};
+// Each chunk's rows are computed in subtasks of up to kQ4Rows rows, and the
+// CTA's chunks are taken in rounds of up to kQ4Round: first every gate
+// subtask of the round (the rows of each chunk half), shared out one at a
+// time to whichever consumer warp asks next; then, once the round's gate
+// values are in, every up subtask (a chunk's gate-active rows, four at a
+// time), shared out the same way; then the chunks are finalized. The
+// subtasks of a phase are independent, so no warp waits on another until
+// the phase ends, and the work is balanced to one subtask. A warp copies
+// the rows of its next subtask (16-byte cp.async per lane, into the other
+// of its two slots) before it computes the current one.
+constexpr int kQ4Round = kMaxLocal;  // chunks per round
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
@@ -1175,13 +1174,16 @@ __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-template <int NT>
+template <int NT, typename Stage>
 __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char* ring, const unsigned char* xb,
-                            const MmaCfg& mc, int i0, int i1, int n_chunks, int cidx, int lane) {
+                            ChunkState<NT>* tab, const MmaCfg& mc, int i0, int i1, int n_chunks, int cidx,
+                            int lane, Stage stage) {
+    constexpr int C = GateUpWarps<NT>::C;
+    const int cthreads = C * kWarp;
     const int d = a.d;
     const int nq = d / 128;  // 32-element groups per K-quarter
     const int g = lane / 4, t = lane % 4;
-    const int wr = g % 4;                  // task row of this lane's A rows
+    const int wr = g % 4;                  // subtask row of this lane's A rows
     const int qa = g / 4, qb = 3 - g / 4;  // their K-quarters
     const bool use_d0 = qa == (t & 1);     // which D element holds this lane's product
     const int qu = use_d0 ? qa : qb;       // the quarter of that product
@@ -1201,44 +1203,88 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
     const unsigned row_bytes = (unsigned)a.row_bytes;
     const int row_chunks = (int)(row_bytes / 16);
     const int n_local = i1 - i0;
-    if (a.test_stall && cidx == 0) {
-        // the failure-detection test: a wait that can only run out (the
-        // other warps take every chunk)
-        warp_wait(&sh.never, 0u, lane, a.status);
-        return;
-    }
+    // the failure-detection test: one warp's wait that can only run out
+    if (a.test_stall && cidx == 0) warp_wait(&sh.never, 0u, lane, a.status);
 
-    // the warp's two chunks: chunk state 2 * cidx + ci
-    int st[2] = {0, 0};           // 0 free, 1 gate rows pending, 2 up rows pending
-    unsigned left[2] = {0u, 0u};  // rows not yet handed to a subtask (gate, then up)
-    int gate_subs[2] = {0, 0};    // gate subtasks not yet computed
-    int up_rows[2] = {0, 0};      // up rows not yet computed
-    int older = 0;                // the chunk claimed first
-    bool more = true;             // chunks may remain to claim
-
-    auto take = [&](unsigned& m) {
-        unsigned sub = 0u;
-        for (int i = 0; i < kQ4Rows && m != 0u; ++i) {
-            sub |= m & (0u - m);
-            m &= m - 1u;
+    // copy a subtask's rows into this warp's slot `slot` (one commit group)
+    auto issue = [&](int kind, int c, unsigned rows, int slot) {
+        volatile ChunkState<NT>& s = tab[c];
+        const int e = s.e;
+        const unsigned char* w = static_cast<const unsigned char*>(kind == kTaskGate ? a.ex[e].wg : a.ex[e].wu);
+        unsigned char* dst = ring + (size_t)(2 * cidx + slot) * kQ4Rows * mc.w_stride;
+        int i = 0;
+        for (unsigned m = rows; m; m &= m - 1u, ++i) {
+            const int j = s.jr[__ffs(m) - 1];
+            const unsigned char* src = w + (size_t)j * row_bytes;
+            unsigned char* drow = dst + (size_t)i * mc.w_stride;
+            for (int k = lane; k < row_chunks; k += kWarp) cp_async16(drow + 16 * k, src + 16 * k);
         }
-        return sub;
+        cp_async_commit();
     };
-    // claim the next chunk with rows into state ci: its rows, expert and local index
-    auto claim = [&](int ci) -> bool {
-        while (more) {
-            int c = 0;
-            if (lane == 0) c = atomicAdd(&sh.next_chunk, 1);
-            c = __shfl_sync(0xffffffffu, c, 0);
-            if (c >= n_local) {
-                more = false;
-                return false;
+    // dot products of the subtask's rows (slot `slot`) with the staged tokens
+    auto compute = [&](int kind, int c, unsigned rows, int slot) {
+        const unsigned char* row = ring + ((size_t)(2 * cidx + slot) * kQ4Rows + wr) * mc.w_stride;
+        const unsigned char* wa = row + qa * (d / 8) + 4 * t;
+        const unsigned char* wb = row + qb * (d / 8) + 4 * t;
+        const unsigned char* sp = row + d / 2 + qu * nq * 2;  // binary16 scales of quarter qu
+        float v0 = 0.0f, v1 = 0.0f;
+#pragma unroll 2
+        for (int G = 0; G < nq; G += 2) {
+            const float2 sc = __half22float2(*reinterpret_cast<const __half2*>(sp + G * 2));
+            const float s0 = (qu & 1) ? sc.y : sc.x;
+            const float s1 = (qu & 1) ? sc.x : sc.y;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                uint32_t b0, b1, b0n, b1n;
+                ldsm_x4(x_col + G * x_step + (h ? x_off1 : x_off0), b0, b1, b0n, b1n);
+                const uint32_t ca = lds32(wa + G * 16 + (h ? a_off1 : a_off0));
+                const uint32_t cb = lds32(wb + G * 16 + (h ? b_off1 : b_off0));
+                // element 8s + 2t + {0, 1} of a group is nibble s (+4) of word t;
+                // the group's two K-steps go to separate accumulators, so the
+                // two MMAs do not wait on each other
+                float dg[4] = {0.0f, 0.0f, 0.0f, 0.0f}, dh[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+                mma_bf16_16816_a4(dg, q4_frag(ca), q4_frag(cb), q4_frag(ca >> 4), q4_frag(cb >> 4), b0, b1);
+                mma_bf16_16816_a4(dh, q4_frag(ca >> 8), q4_frag(cb >> 8), q4_frag(ca >> 12), q4_frag(cb >> 12), b0n,
+                                  b1n);
+                const float pv = use_d0 ? dg[0] + dh[0] : dg[3] + dh[3];
+                if (h == 0)
+                    v0 = fmaf(s0, pv, v0);
+                else
+                    v1 = fmaf(s1, pv, v1);
             }
-            const int item = i0 + c;
+        }
+        // the four K-quarters of (row wr, token t / 2), in the same order in every lane
+        float v = v0 + v1;
+        v += __shfl_xor_sync(0xffffffffu, v, 1);
+        v += __shfl_xor_sync(0xffffffffu, v, 16);
+        volatile ChunkState<NT>& s = tab[c];
+        const int e = s.e;
+        const int ntok = sh.es.ntok[e];
+        if (g < kQ4Rows && (t & 1) == 0 && wr < __popc(rows)) {
+            const int r = __fns(rows, 0, wr + 1);  // chunk row of subtask row wr
+            const int tok = t / 2;
+#pragma unroll
+            for (int k = 0; k < NT; ++k) {
+                const int tk_x = a.route ? sh.es.tok[e][k] : k;
+                if (k < ntok && tk_x == tok) {
+                    if (kind == kTaskGate)
+                        s.g[r][k] = v;
+                    else
+                        s.u[r][k] = v;
+                }
+            }
+        }
+        __syncwarp();
+    };
+
+    // the round's chunks: rows, expert, local index (warp w sets up chunks w, w + C, ...)
+    auto setup = [&](int base, int nr) {
+        for (int c = cidx; c < nr; c += C) {
+            const int item = i0 + base + c;
             const int ea = item / n_chunks;
             const int chunk = item - ea * n_chunks;
             const int e = sh.es.act[ea];
-            volatile ChunkState<NT>& s = sh.cs[2 * cidx + ci];
+            volatile ChunkState<NT>& s = tab[c];
             int j = -1;
             const int p = chunk * kChunk + lane;
             if (lane < kChunk && p < a.n_rows) {
@@ -1257,164 +1303,125 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
             if (lane == 0) {
                 s.e = e;
                 s.chunk = chunk;
-                s.q = c;
-                s.n_gate = __popc(mask);
-                s.gate_cnt = 0;
-                s.up_cnt = 0;
+                s.q = base + c;
+                s.n_gate = (int)mask;  // the chunk's row mask
                 s.gmask = 0u;
             }
-            __syncwarp();
-            if (mask == 0u) {
-                // no rows here: nothing active
-                const int ntok = sh.es.ntok[e];
-                if (lane < ntok) {
-                    const size_t tb = (size_t)(a.bits_tok_base + lane) * a.nbytes;
-                    a.gbits[(size_t)e * a.bits_expert_stride + chunk + tb] = 0;
-                    a.bbits[(size_t)e * a.bits_expert_stride + chunk + tb] = 0;
-                }
-                if (lane == 0) {
-                    a.ubits[(size_t)e * a.nbytes + chunk] = 0;
-                    a.ugbits[(size_t)e * a.nbytes + chunk] = 0;
-                    if (c < kMaxLocal) sh.pd.ub[c] = 0;
-                }
-                continue;
+        }
+        if (cidx == 0 && lane == 0) {
+            sh.q4_ctr[0] = 0;
+            sh.q4_ctr[1] = 0;
+        }
+    };
+    // the next subtask of a phase: chunk c, rows `rows`; false when none is left
+    auto claim = [&](int phase, int n_sub, int& c, unsigned& rows) -> bool {
+        for (;;) {
+            int q = 0;
+            if (lane == 0) q = atomicAdd(&sh.q4_ctr[phase], 1);
+            q = __shfl_sync(0xffffffffu, q, 0);
+            if (q >= n_sub) return false;
+            if (phase == 0) {
+                c = q >> 1;  // gate rows of chunk half q % 2
+                rows = (unsigned)tab[c].n_gate & (0xFu << (4 * (q & 1)));
+                if (rows == 0u) continue;
+            } else {
+                const unsigned ent = sh.q4_up[q];
+                c = (int)(ent >> 8);
+                rows = ent & 0xFFu;
             }
-            st[ci] = 1;
-            left[ci] = mask;
-            gate_subs[ci] = (__popc(mask) + kQ4Rows - 1) / kQ4Rows;
-            older = st[ci ^ 1] != 0 ? (ci ^ 1) : ci;
             return true;
         }
-        return false;
     };
-    // the next subtask: the up rows of a finished gate (older chunk first),
-    // else pending gate rows, else a newly claimed chunk's first gate rows
-    auto pick = [&]() -> Q4Sub {
-        for (int k = 0; k < 2; ++k) {
-            const int ci = k == 0 ? older : older ^ 1;
-            if (st[ci] == 2 && left[ci] != 0u) return Q4Sub{kTaskUp, ci, take(left[ci])};
-        }
-        for (int k = 0; k < 2; ++k) {
-            const int ci = k == 0 ? older : older ^ 1;
-            if (st[ci] == 1 && left[ci] != 0u) return Q4Sub{kTaskGate, ci, take(left[ci])};
-        }
-        for (int ci = 0; ci < 2; ++ci)
-            if (st[ci] == 0 && claim(ci)) return Q4Sub{kTaskGate, ci, take(left[ci])};
-        return Q4Sub{kTaskEnd, 0, 0u};
-    };
-    // copy a subtask's rows into this warp's slot `slot` (one commit group)
-    auto issue = [&](const Q4Sub& sb, int slot) {
-        volatile ChunkState<NT>& s = sh.cs[2 * cidx + sb.ci];
-        const int e = s.e;
-        const unsigned char* w = static_cast<const unsigned char*>(sb.kind == kTaskGate ? a.ex[e].wg : a.ex[e].wu);
-        unsigned char* dst = ring + (size_t)(2 * cidx + slot) * kQ4Rows * mc.w_stride;
-        int i = 0;
-        for (unsigned m = sb.rows; m; m &= m - 1u, ++i) {
-            const int j = s.jr[__ffs(m) - 1];
-            const unsigned char* src = w + (size_t)j * row_bytes;
-            unsigned char* drow = dst + (size_t)i * mc.w_stride;
-            for (int c = lane; c < row_chunks; c += kWarp) cp_async16(drow + 16 * c, src + 16 * c);
-        }
-        cp_async_commit();
-    };
+    // The weights do not depend on the activations: the first round's
+    // chunks and each warp's first gate rows are set going before the
+    // activations are staged (and, for the dense layer, before the wait for
+    // the kernel that writes them).
+    int c_first = 0;
+    unsigned r_first = 0u;
+    setup(0, min(kQ4Round, n_local));
+    named_bar_sync(1, cthreads);
+    const bool have_first = claim(0, 2 * min(kQ4Round, n_local), c_first, r_first);
+    if (have_first) issue(kTaskGate, c_first, r_first, 0);
+    stage();
 
-    Q4Sub cur = pick();
-    int slot = 0;
-    if (cur.kind != kTaskEnd) issue(cur, slot);
-    while (cur.kind != kTaskEnd) {
-        const Q4Sub nxt = pick();
-        if (nxt.kind != kTaskEnd) {
-            issue(nxt, slot ^ 1);
-            cp_async_wait<1>();
-        } else {
-            cp_async_wait<0>();
+    for (int base = 0; base < n_local; base += kQ4Round) {
+        const int nr = min(kQ4Round, n_local - base);
+        if (base > 0) {
+            setup(base, nr);
+            named_bar_sync(1, cthreads);
         }
-        __syncwarp();  // every lane's copies of the current subtask have landed
-        const unsigned char* row = ring + ((size_t)(2 * cidx + slot) * kQ4Rows + wr) * mc.w_stride;
-        const unsigned char* wa = row + qa * (d / 8) + 4 * t;
-        const unsigned char* wb = row + qb * (d / 8) + 4 * t;
-        const unsigned char* sp = row + d / 2 + qu * nq * 2;  // binary16 scales of quarter qu
-        float v0 = 0.0f, v1 = 0.0f;
-#pragma unroll 2
-        for (int G = 0; G < nq; G += 2) {
-            const float2 sc = __half22float2(*reinterpret_cast<const __half2*>(sp + G * 2));
-            const float s0 = (qu & 1) ? sc.y : sc.x;
-            const float s1 = (qu & 1) ? sc.x : sc.y;
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                uint32_t b0, b1, b0n, b1n;
-                ldsm_x4(x_col + G * x_step + (h ? x_off1 : x_off0), b0, b1, b0n, b1n);
-                const uint32_t ca = lds32(wa + G * 16 + (h ? a_off1 : a_off0));
-                const uint32_t cb = lds32(wb + G * 16 + (h ? b_off1 : b_off0));
-                float dg[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-                // element 8s + 2t + {0, 1} of a group is nibble s (+4) of word t
-                mma_bf16_16816_a4(dg, q4_frag(ca), q4_frag(cb), q4_frag(ca >> 4), q4_frag(cb >> 4), b0, b1);
-                mma_bf16_16816_a4(dg, q4_frag(ca >> 8), q4_frag(cb >> 8), q4_frag(ca >> 12), q4_frag(cb >> 12), b0n,
-                                  b1n);
-                const float pv = use_d0 ? dg[0] : dg[3];
-                if (h == 0)
-                    v0 = fmaf(s0, pv, v0);
-                else
-                    v1 = fmaf(s1, pv, v1);
+        for (int phase = 0; phase < 2; ++phase) {
+            const int kind = phase == 0 ? kTaskGate : kTaskUp;
+            const int n_sub = phase == 0 ? 2 * nr : sh.q4_ctr[2];
+            int c_cur = 0, c_nxt = 0;
+            unsigned r_cur = 0u, r_nxt = 0u;
+            bool have;
+            int slot = 0;
+            if (base == 0 && phase == 0) {
+                have = have_first;
+                c_cur = c_first;
+                r_cur = r_first;
+            } else {
+                have = claim(phase, n_sub, c_cur, r_cur);
+                if (have) issue(kind, c_cur, r_cur, slot);
             }
-        }
-        // the four K-quarters of (row wr, token t / 2), in the same order in every lane
-        float v = v0 + v1;
-        v += __shfl_xor_sync(0xffffffffu, v, 1);
-        v += __shfl_xor_sync(0xffffffffu, v, 16);
-        const int ci = cur.ci;
-        const int cs_i = 2 * cidx + ci;
-        volatile ChunkState<NT>& s = sh.cs[cs_i];
-        const int e = s.e;
-        const int ntok = sh.es.ntok[e];
-        if (g < kQ4Rows && (t & 1) == 0 && wr < __popc(cur.rows)) {
-            const int r = __fns(cur.rows, 0, wr + 1);  // chunk row of task row wr
-            const int tok = t / 2;
-#pragma unroll
-            for (int k = 0; k < NT; ++k) {
-                const int tk_x = a.route ? sh.es.tok[e][k] : k;
-                if (k < ntok && tk_x == tok) {
-                    if (cur.kind == kTaskGate)
-                        s.g[r][k] = v;
-                    else
-                        s.u[r][k] = v;
+            while (have) {
+                const bool have_nxt = claim(phase, n_sub, c_nxt, r_nxt);
+                if (have_nxt) {
+                    issue(kind, c_nxt, r_nxt, slot ^ 1);
+                    cp_async_wait<1>();
+                } else {
+                    cp_async_wait<0>();
                 }
+                __syncwarp();  // every lane's copies of the current subtask have landed
+                compute(kind, c_cur, r_cur, slot);
+                c_cur = c_nxt;
+                r_cur = r_nxt;
+                have = have_nxt;
+                slot ^= 1;
             }
-        }
-        __syncwarp();
-        bool done = false;
-        if (cur.kind == kTaskGate) {
-            if (--gate_subs[ci] == 0) {
-                // every gate row of the chunk is in: which rows need their W_up row?
-                bool ga = false;
-                if (lane < kChunk && s.jr[lane] >= 0) {
+            named_bar_sync(1, cthreads);
+            if (phase == 0 && cidx == 0) {
+                // gate-active rows of each chunk (lane c), and the up subtasks:
+                // the first four of them, then the rest
+                unsigned gm = 0u;
+                if (lane < nr) {
+                    volatile ChunkState<NT>& s = tab[lane];
+                    const int ntok = sh.es.ntok[s.e];
+                    for (int r = 0; r < kChunk; ++r) {
+                        bool ga = false;
+                        if (s.jr[r] >= 0) {
 #pragma unroll
-                    for (int k = 0; k < NT; ++k) ga |= (k < ntok) && (s.g[lane][k] > 0.0f);
+                            for (int k = 0; k < NT; ++k) ga |= (k < ntok) && (s.g[r][k] > 0.0f);
+                        }
+                        if (ga) gm |= 1u << r;
+                    }
+                    s.gmask = gm;
                 }
-                const unsigned gm = __ballot_sync(0xffffffffu, ga);
-                if (lane == 0) s.gmask = gm;
+                const int cnt = __popc(gm) > kQ4Rows ? 2 : (gm != 0u ? 1 : 0);
+                int incl = cnt;
+#pragma unroll
+                for (int o = 1; o < kWarp; o <<= 1) {
+                    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += v;
+                }
+                int pos = incl - cnt;
+                unsigned m = gm;
+                for (int k = 0; k < cnt; ++k) {
+                    unsigned sub = 0u;
+                    for (int i = 0; i < kQ4Rows && m != 0u; ++i) {
+                        sub |= m & (0u - m);
+                        m &= m - 1u;
+                    }
+                    sh.q4_up[pos++] = ((unsigned)lane << 8) | sub;
+                }
+                if (lane == kWarp - 1) sh.q4_ctr[2] = incl;
                 __syncwarp();
-                st[ci] = 2;
-                left[ci] = gm;
-                up_rows[ci] = __popc(gm);
-                done = gm == 0u;
             }
-        } else {
-            up_rows[ci] -= __popc(cur.rows);
-            done = up_rows[ci] == 0;
+            if (phase == 0) named_bar_sync(1, cthreads);
         }
-        if (done) {
-            finalize_chunk<NT>(a, sh, cs_i, lane);
-            st[ci] = 0;
-            older = ci ^ 1;
-        }
-        cur = nxt;
-        slot ^= 1;
-        if (cur.kind == kTaskEnd) {
-            // up rows of a chunk whose gate finished just now may still be due
-            cur = pick();
-            if (cur.kind != kTaskEnd) issue(cur, slot);
-        }
+        for (int c = cidx; c < nr; c += C) finalize_chunk_s<NT>(a, sh, tab[c], lane);
+        named_bar_sync(1, cthreads);  // the table is refilled next round
     }
 }
 
@@ -1424,10 +1431,11 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
     constexpr int C = GateUpWarps<NT>::C;
     __shared__ GateUpShared<NT> sh;
     extern __shared__ __align__(128) unsigned char dyn[];
-    // [NT][4 quarters][d/4 bf16 + pad] activations
+    // [NT][4 quarters][d/4 bf16 + pad] activations, the ring, the round's chunks
     unsigned char* xb = dyn;
     const size_t x_bytes = ((size_t)kAccMaxTokens * mc.x_stride + 127) / 128 * 128;
     unsigned char* ring = dyn + x_bytes;  // [C][2 slots][kQ4Rows][w_stride]
+    ChunkState<NT>* tab = reinterpret_cast<ChunkState<NT>*>(ring + (size_t)mc.groups * kQ4Rows * mc.w_stride);
     const int n_x = a.route ? a.batch : a.nt;
 
     const int lane = threadIdx.x & 31;
@@ -1435,8 +1443,6 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
     if (threadIdx.x == 0) {
         mbar_init(&sh.never, 1);
         for (int q = 0; q < kMaxLocal; ++q) sh.pd.ub[q] = 0;
-        for (int w = 0; w < 2 * kWindow; ++w) mbar_init(&sh.chunk_free[w], 1);
-        sh.next_chunk = 0;
         mbar_fence_init();
     }
     const bool early = a.rows == nullptr && a.route == nullptr;
@@ -1450,12 +1456,13 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
     const int i1 = (int)((long long)n_items * (blockIdx.x + 1) / gridDim.x);
 
     if (warp == 0) return;  // the consumer warps copy their own rows
-    if (early) pdl_wait();
     const int ctid = threadIdx.x - kWarp;
     const int cthreads = C * kWarp;
     const int x_tok0 = a.route ? 0 : a.tok0;
     const int dq = a.d / 4;
     auto xpos = [&](int i) { return (i / dq) * (dq + kQ4QuarterPad / 2) + i % dq; };  // bf16 index in a row
+    auto stage = [&]() {
+    if (early) pdl_wait();
     for (int t = 0; t < NT; ++t) {
         __nv_bfloat16* xrow = reinterpret_cast<__nv_bfloat16*>(xb + (size_t)t * mc.x_stride);
         if (t >= n_x) {
@@ -1480,14 +1487,13 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
         }
     }
     named_bar_sync(1, cthreads);
-    consume_q4w<NT>(a, sh, ring, xb, mc, i0, i1, n_chunks, warp - 1, lane);
-    // every chunk is finalized once all consumers are here
-    named_bar_sync(1, cthreads);
+    };
+    consume_q4w<NT>(a, sh, ring, xb, tab, mc, i0, i1, n_chunks, warp - 1, lane, stage);
     down_partial<T, NT, true>(a, sh, i0, i1, n_chunks, warp - 1, lane);
 }
 
 // Shared memory of the INT4 kernel: activations (kAccMaxTokens rows of four
-// padded K-quarters), then the ring. A slot row's stride is
+// padded K-quarters), the ring, and the states of a round's chunks. A slot row's stride is
 // 32 bytes past a multiple of 128, which with the swapped order of odd
 // quarters puts the 32 lanes' code words in 32 banks.
 static size_t q4w_smem(int d, int avail, MmaCfg* mc) {
@@ -1501,7 +1507,7 @@ static size_t q4w_smem(int d, int avail, MmaCfg* mc) {
     mc->lookahead = 0;
     mc->end_tasks = 0;
     (void)avail;
-    return x_bytes + (size_t)mc->groups * slot;
+    return x_bytes + (size_t)mc->groups * slot + (size_t)kQ4Round * sizeof(ChunkState<kAccMaxTokens>);
 }
 
 // ---------------------------------------------------------------------------
