@@ -1139,11 +1139,6 @@ __device__ __forceinline__ uint32_t q4_frag(uint32_t v) {
     p = __hsub2(p, __floats2bfloat162_rn(136.0f, 136.0f));
     return *reinterpret_cast<const uint32_t*>(&p);
 }
-__device__ __forceinline__ uint32_t lds32(const void* p) {
-    uint32_t v;
-    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(smem_u32(p)));
-    return v;
-}
 // d += A * B for one m16n8k16 step with all 16 A rows.
 __device__ __forceinline__ void mma_bf16_16816_a4(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
                                                   uint32_t b0, uint32_t b1) {
@@ -1187,10 +1182,15 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
     const int qa = g / 4, qb = 3 - g / 4;  // their K-quarters
     const bool use_d0 = qa == (t & 1);     // which D element holds this lane's product
     const int qu = use_d0 ? qa : qb;       // the quarter of that product
-    // A words: word t of each group of the lane's two quarters; odd quarters
-    // take the pair (G, G + 1) in the order (G + 1, G)
-    const int a_off0 = (qa & 1) * 16, a_off1 = 16 - a_off0;
-    const int b_off0 = (qb & 1) * 16, b_off1 = 16 - b_off0;
+    // A words: word t of each group of the lane's two quarters, for a pair
+    // of groups (G, G + 1) at once by ldmatrix: this lane addresses row
+    // lane % 8 of matrix lane / 8, i.e. the 16 code bytes of subtask row
+    // (lane % 8) % 4 in quarter qa (matrices 0, 2) or qb (1, 3) of group G
+    // (matrices 0, 1) or G + 1 (2, 3); odd quarters take the pair in the
+    // order (G + 1, G).
+    const int lg = lane % 8, lm = lane / 8;
+    const int l_q = (lm & 1) ? 3 - lg / 4 : lg / 4;
+    const int l_off = l_q * (d / 8) + (((lm >> 1) ^ (l_q & 1)) * 16);
     // B: this lane addresses column n = lane % 8 for ldmatrix; with one
     // token, columns 4-7 repeat token 0 (same addresses, no bank conflict)
     // and their products are not used
@@ -1223,9 +1223,9 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
     };
     // dot products of the subtask's rows (slot `slot`) with the staged tokens
     auto compute = [&](int kind, int c, unsigned rows, int slot) {
-        const unsigned char* row = ring + ((size_t)(2 * cidx + slot) * kQ4Rows + wr) * mc.w_stride;
-        const unsigned char* wa = row + qa * (d / 8) + 4 * t;
-        const unsigned char* wb = row + qb * (d / 8) + 4 * t;
+        const unsigned char* sbase = ring + (size_t)(2 * cidx + slot) * kQ4Rows * mc.w_stride;
+        const unsigned char* row = sbase + (size_t)wr * mc.w_stride;
+        const uint32_t c_addr = smem_u32(sbase + (size_t)(lg % 4) * mc.w_stride + l_off);
         const unsigned char* sp = row + d / 2 + qu * nq * 2;  // binary16 scales of quarter qu
         float v0 = 0.0f, v1 = 0.0f;
 #pragma unroll 2
@@ -1233,12 +1233,14 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
             const float2 sc = __half22float2(*reinterpret_cast<const __half2*>(sp + G * 2));
             const float s0 = (qu & 1) ? sc.y : sc.x;
             const float s1 = (qu & 1) ? sc.x : sc.y;
+            uint32_t cw[4];  // (qa, G), (qb, G), (qa, G + 1), (qb, G + 1) in this lane's order
+            ldsm_x4(c_addr + G * 16, cw[0], cw[1], cw[2], cw[3]);
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
                 uint32_t b0, b1, b0n, b1n;
                 ldsm_x4(x_col + G * x_step + (h ? x_off1 : x_off0), b0, b1, b0n, b1n);
-                const uint32_t ca = lds32(wa + G * 16 + (h ? a_off1 : a_off0));
-                const uint32_t cb = lds32(wb + G * 16 + (h ? b_off1 : b_off0));
+                const uint32_t ca = cw[2 * h];
+                const uint32_t cb = cw[2 * h + 1];
                 // element 8s + 2t + {0, 1} of a group is nibble s (+4) of word t;
                 // the group's two K-steps go to separate accumulators, so the
                 // two MMAs do not wait on each other
@@ -1511,6 +1513,290 @@ static size_t q4w_smem(int d, int avail, MmaCfg* mc) {
 }
 
 // ---------------------------------------------------------------------------
+// bf16 rows, passes of 1-2 tokens, without a producer thread. A single
+// thread issuing one bulk copy per row sustains only about 3.7 TB/s for
+// 8 KB rows, so here every consumer warp copies its own rows (16-byte
+// cp.async per lane) into its own ring slots, a few rows ahead of the one it
+// computes. The CTA's chunks are taken in rounds, as in the INT4 kernel:
+// every gate row of the round is handed to whichever warp asks next, then
+// every gate-active up row, then the chunks are finalized.
+// ---------------------------------------------------------------------------
+constexpr int kRowsMaxAhead = 2;  // rows a warp has in flight besides the one it computes
+
+struct RowsCfg {
+    int xs_stride;   // floats per activation row in shared memory
+    int slot_bytes;  // bytes per ring slot: one row, rounded up to 128
+    int ahead;       // rows in flight per warp besides the current one (1 or 2)
+};
+
+template <int N>
+__device__ __forceinline__ void cp_async_wait_n(int n) {
+    // wait until at most n of this thread's copy groups are pending (n <= N)
+    if (n <= 0) {
+        cp_async_wait<0>();
+    } else if (n == 1 || N == 1) {
+        cp_async_wait<1>();
+    } else {
+        cp_async_wait<2>();
+    }
+}
+
+template <typename T, int NT, typename Stage>
+__device__ void consume_rows(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char* ring, const float* xs,
+                             ChunkState<NT>* tab, unsigned short* ulist, const RowsCfg& rc, int i0, int i1,
+                             int n_chunks, int cidx, int lane, Stage stage) {
+    constexpr int C = GateUpWarps<NT>::C;
+    const int cthreads = C * kWarp;
+    const unsigned row_bytes = (unsigned)(a.d * sizeof(T));
+    const int row_chunks = (int)(row_bytes / 16);
+    const int n_local = i1 - i0;
+    const int P = rc.ahead + 1;  // this warp's slots
+    // the failure-detection test: one warp's wait that can only run out
+    if (a.test_stall && cidx == 0) warp_wait(&sh.never, 0u, lane, a.status);
+
+    auto setup = [&](int base, int nr) {
+        for (int c = cidx; c < nr; c += C) {
+            const int item = i0 + base + c;
+            const int ea = item / n_chunks;
+            const int chunk = item - ea * n_chunks;
+            const int e = sh.es.act[ea];
+            volatile ChunkState<NT>& s = tab[c];
+            int j = -1;
+            const int p = chunk * kChunk + lane;
+            if (lane < kChunk && p < a.n_rows) {
+                if (a.rows != nullptr) {
+                    const int jj = a.rows[p];
+                    if ((unsigned)jj < (unsigned)a.m && (p == 0 || a.rows[p - 1] < jj))
+                        j = jj;
+                    else
+                        atomicOr(a.status, kStatusBadIndex);
+                } else {
+                    j = p;
+                }
+            }
+            if (lane < kChunk) s.jr[lane] = j;
+            const unsigned mask = __ballot_sync(0xffffffffu, j >= 0);
+            if (lane == 0) {
+                s.e = e;
+                s.chunk = chunk;
+                s.q = base + c;
+                s.n_gate = (int)mask;  // the chunk's row mask
+                s.gmask = 0u;
+            }
+        }
+        if (cidx == 0 && lane == 0) {
+            sh.q4_ctr[0] = 0;
+            sh.q4_ctr[1] = 0;
+        }
+    };
+    // the next row of a phase: chunk c, row r; false when none is left
+    auto claim = [&](int phase, int n_sub, int& c, int& r) -> bool {
+        for (;;) {
+            int q = 0;
+            if (lane == 0) q = atomicAdd(&sh.q4_ctr[phase], 1);
+            q = __shfl_sync(0xffffffffu, q, 0);
+            if (q >= n_sub) return false;
+            if (phase == 0) {
+                c = q / kChunk;
+                r = q % kChunk;
+                if ((((unsigned)tab[c].n_gate >> r) & 1u) == 0u) continue;
+            } else {
+                const unsigned ent = ulist[q];
+                c = (int)(ent / kChunk);
+                r = (int)(ent % kChunk);
+            }
+            return true;
+        }
+    };
+    auto issue = [&](int kind, int c, int r, int slot) {
+        volatile ChunkState<NT>& s = tab[c];
+        const int e = s.e;
+        const unsigned char* w = static_cast<const unsigned char*>(kind == kTaskGate ? a.ex[e].wg : a.ex[e].wu);
+        const unsigned char* src = w + (size_t)s.jr[r] * row_bytes;
+        unsigned char* dst = ring + (size_t)(cidx * P + slot) * rc.slot_bytes;
+        for (int k = lane; k < row_chunks; k += kWarp) cp_async16(dst + 16 * k, src + 16 * k);
+        cp_async_commit();
+    };
+    auto compute = [&](int kind, int c, int r, int slot) {
+        volatile ChunkState<NT>& s = tab[c];
+        const int e = s.e;
+        const int ntok = sh.es.ntok[e];
+        int xt[NT];
+#pragma unroll
+        for (int k = 0; k < NT; ++k) xt[k] = k < ntok ? (a.route ? sh.es.tok[e][k] : k) : 0;
+        float acc[NT];
+        smem_row_dot<T, NT>(ring + (size_t)(cidx * P + slot) * rc.slot_bytes, xs, rc.xs_stride, xt, ntok, a.d,
+                            lane, acc);
+        if (lane == 0) {
+            volatile float* dst = kind == kTaskGate ? s.g[r] : s.u[r];
+#pragma unroll
+            for (int k = 0; k < NT; ++k) dst[k] = acc[k];
+        }
+        __syncwarp();
+    };
+
+    // The weights do not depend on the activations: the first round's rows
+    // are set going before the activations are staged (and, for the dense
+    // layer, before the wait for the kernel that writes them).
+    int qc[kRowsMaxAhead + 1], qr[kRowsMaxAhead + 1];  // claimed rows, oldest first
+    int n_q = 0, head_slot = 0;
+    const int nr0 = min(kQ4Round, n_local);
+    setup(0, nr0);
+    named_bar_sync(1, cthreads);
+    while (n_q < P && claim(0, kChunk * nr0, qc[n_q], qr[n_q])) {
+        issue(kTaskGate, qc[n_q], qr[n_q], n_q);
+        ++n_q;
+    }
+    stage();
+
+    for (int base = 0; base < n_local; base += kQ4Round) {
+        const int nr = min(kQ4Round, n_local - base);
+        if (base > 0) {
+            setup(base, nr);
+            named_bar_sync(1, cthreads);
+        }
+        for (int phase = 0; phase < 2; ++phase) {
+            const int kind = phase == 0 ? kTaskGate : kTaskUp;
+            const int n_sub = phase == 0 ? kChunk * nr : sh.q4_ctr[2];
+            if (!(base == 0 && phase == 0)) {
+                n_q = 0;
+                head_slot = 0;
+                while (n_q < P && claim(phase, n_sub, qc[n_q], qr[n_q])) {
+                    issue(kind, qc[n_q], qr[n_q], n_q);
+                    ++n_q;
+                }
+            }
+            while (n_q > 0) {
+                cp_async_wait_n<kRowsMaxAhead>(n_q - 1);  // the oldest row has landed
+                __syncwarp();
+                compute(kind, qc[0], qr[0], head_slot);
+                // its slot takes the next row
+                for (int i = 1; i < n_q; ++i) {
+                    qc[i - 1] = qc[i];
+                    qr[i - 1] = qr[i];
+                }
+                --n_q;
+                const int free_slot = head_slot;
+                head_slot = head_slot + 1 == P ? 0 : head_slot + 1;
+                if (claim(phase, n_sub, qc[n_q], qr[n_q])) {
+                    issue(kind, qc[n_q], qr[n_q], free_slot);
+                    ++n_q;
+                }
+            }
+            named_bar_sync(1, cthreads);
+            if (phase == 0 && cidx == 0) {
+                // gate-active rows of each chunk (lane c), listed in chunk order
+                unsigned gm = 0u;
+                if (lane < nr) {
+                    volatile ChunkState<NT>& s = tab[lane];
+                    const int ntok = sh.es.ntok[s.e];
+                    for (int r = 0; r < kChunk; ++r) {
+                        bool ga = false;
+                        if (s.jr[r] >= 0) {
+#pragma unroll
+                            for (int k = 0; k < NT; ++k) ga |= (k < ntok) && (s.g[r][k] > 0.0f);
+                        }
+                        if (ga) gm |= 1u << r;
+                    }
+                    s.gmask = gm;
+                }
+                const int cnt = __popc(gm);
+                int incl = cnt;
+#pragma unroll
+                for (int o = 1; o < kWarp; o <<= 1) {
+                    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += v;
+                }
+                int pos = incl - cnt;
+                for (unsigned m = gm; m; m &= m - 1u) ulist[pos++] = (unsigned short)(lane * kChunk + __ffs(m) - 1);
+                if (lane == kWarp - 1) sh.q4_ctr[2] = incl;
+                __syncwarp();
+            }
+            if (phase == 0) named_bar_sync(1, cthreads);
+        }
+        for (int c = cidx; c < nr; c += C) finalize_chunk_s<NT>(a, sh, tab[c], lane);
+        named_bar_sync(1, cthreads);  // the table is refilled next round
+    }
+}
+
+template <typename T, int NT>
+__global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(const FfnLaunch a, const RowsCfg rc) {
+    constexpr int C = GateUpWarps<NT>::C;
+    __shared__ GateUpShared<NT> sh;
+    extern __shared__ __align__(128) unsigned char dyn[];
+    float* xs = reinterpret_cast<float*>(dyn);  // [NT][xs_stride]
+    unsigned char* ring = dyn + (size_t)NT * rc.xs_stride * sizeof(float);  // [C][ahead + 1][slot_bytes]
+    ChunkState<NT>* tab =
+        reinterpret_cast<ChunkState<NT>*>(ring + (size_t)C * (rc.ahead + 1) * rc.slot_bytes);
+    unsigned short* ulist = reinterpret_cast<unsigned short*>(tab + kQ4Round);  // [kQ4Round * kChunk]
+    const int n_x = a.route ? a.batch : a.nt;
+
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    if (threadIdx.x == 0) {
+        mbar_init(&sh.never, 1);
+        for (int q = 0; q < kMaxLocal; ++q) sh.pd.ub[q] = 0;
+        mbar_fence_init();
+    }
+    const bool early = a.rows == nullptr && a.route == nullptr;
+    if (!early) pdl_wait();
+    resolve_experts(a, sh.es);
+    pdl_launch_dependents();
+
+    const int n_chunks = (a.n_rows + kChunk - 1) / kChunk;
+    const int n_items = sh.es.n_act * n_chunks;
+    const int i0 = (int)((long long)n_items * blockIdx.x / gridDim.x);
+    const int i1 = (int)((long long)n_items * (blockIdx.x + 1) / gridDim.x);
+
+    if (warp == 0) return;  // the consumer warps copy their own rows
+    const int ctid = threadIdx.x - kWarp;
+    const int cthreads = C * kWarp;
+    const int x_tok0 = a.route ? 0 : a.tok0;
+    auto stage = [&]() {
+        if (early) pdl_wait();
+        for (int t = 0; t < n_x; ++t) {
+            float* xrow = xs + (size_t)t * rc.xs_stride;
+            if (a.norm_from_h) {
+                const float* hr = a.h + (size_t)(x_tok0 + t) * a.d;
+                float ss = 0.0f;
+                for (int i = ctid; i < a.d; i += cthreads) ss = fmaf(hr[i], hr[i], ss);
+                ss = warp_sum(ss);
+                if (lane == 0) sh.red[warp - 1] = ss;
+                named_bar_sync(1, cthreads);
+                float tot = 0.0f;
+                for (int w = 0; w < C; ++w) tot += sh.red[w];
+                const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)a.d), 1e-5f));
+                for (int i = ctid; i < a.d; i += cthreads)
+                    xrow[xs_index<T>(i)] = (i == a.d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hr[i], rms));
+                named_bar_sync(1, cthreads);
+            } else {
+                for (int i = ctid; i < a.d; i += cthreads)
+                    xrow[xs_index<T>(i)] = Vec<T>::load1(a.x, (size_t)(x_tok0 + t) * a.d + i);
+            }
+        }
+        named_bar_sync(1, cthreads);
+    };
+    consume_rows<T, NT>(a, sh, ring, xs, tab, ulist, rc, i0, i1, n_chunks, warp - 1, lane, stage);
+    down_partial<T, NT>(a, sh, i0, i1, n_chunks, warp - 1, lane);
+}
+
+// Shared memory of the copy-by-consumer kernel: activations, the ring (as
+// many rows ahead per warp as fit, up to kRowsMaxAhead), a round's chunk
+// states and its list of up rows.
+static size_t rows_smem(int elem, int d, int nt, int avail, RowsCfg* rc) {
+    rc->xs_stride = (d + 255) / 256 * 256;
+    rc->slot_bytes = (d * elem + 127) / 128 * 128;
+    const size_t fixed = (size_t)nt * rc->xs_stride * sizeof(float) +
+                         (size_t)kQ4Round * sizeof(ChunkState<kAccMaxTokens>) +
+                         (size_t)kQ4Round * kChunk * sizeof(unsigned short);
+    const int C = GateUpWarps<1>::C;
+    int ahead = kRowsMaxAhead;
+    while (ahead > 1 && fixed + (size_t)C * (ahead + 1) * rc->slot_bytes > (size_t)avail) --ahead;
+    rc->ahead = ahead;
+    return fixed + (size_t)C * (ahead + 1) * rc->slot_bytes;
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 int gate_up_config(int wdtype, int d, int x_tokens, int optin_smem, int* slots, int* slot_bytes,
@@ -1593,6 +1879,34 @@ static cudaError_t launch_q4w_t(const FfnLaunch& a, int grid, cudaStream_t strea
     return cudaLaunchKernelEx(&lc, k_gate_up_q4w<NT>, a, mc);
 }
 
+template <typename T, int NT>
+static cudaError_t launch_rows_t(const FfnLaunch& a, int grid, cudaStream_t stream, bool pdl) {
+    RowsCfg rc;
+    const size_t smem = rows_smem((int)sizeof(T), a.d, NT, g_optin - kSmemMargin, &rc);
+    if (smem + kSmemMargin > (size_t)g_optin) return cudaErrorInvalidValue;
+    const int n_x = a.route ? a.batch : a.nt;
+    if (n_x > NT || a.partial == nullptr || a.partial_slots < n_x || a.partial_ctas < grid)
+        return cudaErrorInvalidValue;
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(GateUpWarps<NT>::THREADS);
+    lc.dynamicSmemBytes = smem;
+    lc.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&lc, k_gate_up_rows<T, NT>, a, rc);
+}
+
+// bf16 passes of 1-2 tokens take the copy-by-consumer kernel when its ring fits
+static bool use_rows(int wdtype, int d, int pass_tokens) {
+    RowsCfg rc;
+    return wdtype == 1 && pass_tokens <= kAccMaxTokens &&
+           rows_smem(2, d, pass_tokens, g_optin - kSmemMargin, &rc) + kSmemMargin <= (size_t)g_optin;
+}
+
 constexpr int kMmaMinTokens = 4;  // narrowest bf16 pass that takes the tensor-core variant
 
 static bool use_mma(int wdtype, int d, int pass_tokens) {
@@ -1630,6 +1944,8 @@ cudaError_t prepare_gate_up(int optin_smem) {
     const int dyn = optin_smem - kSmemMargin;
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_rows<__nv_bfloat16, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_rows<__nv_bfloat16, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_q4w<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_q4w<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     return e;
@@ -1643,6 +1959,10 @@ cudaError_t launch_gate_up(const FfnLaunch& a, int wdtype, int pass_tokens, int 
         if (pass_tokens == 1) return launch_q4w_t<1>(a, grid, stream, pdl);
         if (pass_tokens == 2) return launch_q4w_t<2>(a, grid, stream, pdl);
         return cudaErrorInvalidValue;
+    }
+    if (use_rows(wdtype, a.d, pass_tokens)) {
+        if (pass_tokens == 1) return launch_rows_t<__nv_bfloat16, 1>(a, grid, stream, pdl);
+        if (pass_tokens == 2) return launch_rows_t<__nv_bfloat16, 2>(a, grid, stream, pdl);
     }
     if (use_mma(wdtype, a.d, pass_tokens)) {
         if (pass_tokens == 4) return launch_mma_t<4>(a, grid, stream, pdl);
