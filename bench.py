@@ -42,14 +42,15 @@ UNIT = "tokens/s"
 NOMINAL_HBM_GBS = 7900.0
 
 
-# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one k_gate_up
-# launch on one full-size layer of the batch-1 stack, from the ncu capture
-# summarised in profiles/k_gate_up-k_down-mistral7b-layer-full.md, and the
-# SHA-256 of the kernel sources it was taken on: once they change, the figure
-# no longer describes the kernel and is reported as null.
-NCU_TRAFFIC = {"bytes": 166.09e6,
-               "sources": ("paper_2406_05955_gb300/csrc/ts_gate_up.cu", "paper_2406_05955_gb300/csrc/ts_kernels.cuh"),
-               "sha256": "50374b962222bce7cc6e72c883b9becb4eb94cdc0a3984ef8e3c4d4be5838de3"}
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one gate+up
+# launch on one full-size layer of the batch-1 stacks (bf16 rows: k_gate_up_rows;
+# INT4 rows: k_gate_up_q4w), from one ncu capture each, and the SHA-256 of the
+# kernel sources they were taken on: once those change, the figures no longer
+# describe the kernels and are reported as null.
+KERNEL_SOURCES = ("paper_2406_05955_gb300/csrc/ts_gate_up.cu", "paper_2406_05955_gb300/csrc/ts_kernels.cuh")
+NCU_TRAFFIC = {"bytes": {"bf16": 165.28e6, "int4": 45.69e6},
+               "sources": KERNEL_SOURCES,
+               "sha256": "1bbecbfd3a66fdc2944049b17bf75ed5d35ccf545aa4dbf83361b16bf81e8fb8"}
 
 
 def kernel_sources_sha256(paths) -> str:
@@ -60,12 +61,12 @@ def kernel_sources_sha256(paths) -> str:
     return h.hexdigest()
 
 
-def ncu_traffic() -> float | None:
+def ncu_traffic(kind: str) -> float | None:
     try:
         ok = kernel_sources_sha256(NCU_TRAFFIC["sources"]) == NCU_TRAFFIC["sha256"]
     except OSError:
         ok = False
-    return NCU_TRAFFIC["bytes"] if ok else None
+    return NCU_TRAFFIC["bytes"][kind] if ok else None
 
 
 def load_peaks() -> dict:
@@ -409,11 +410,12 @@ def run_ours(args, dist: Dist) -> dict | None:
             "both_active_per_layer": statistics.mean(c[1] for c in nb["per_layer_counts"]),
         },
         "roofline": {"bound": "hbm",
-                     "kernel": ("k_gate_up (gate GEMV, gathered up projection, this CTA's share of the "
-                                "down projection)" if B <= 2 else "k_gate_up (gate GEMV + gathered up projection)"),
+                     "kernel": (("k_gate_up_q4w" if int4 else "k_gate_up_rows") +
+                                " (gate GEMV, gathered up projection, this CTA's share of the down projection)"
+                                if B <= 2 else "k_gate_up_mma (gate GEMM + gathered up projection)"),
                      "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                      "frac": achieved / peaks["hbm_gbs"], "peak_source": peaks["source"],
-                     "traffic": None if predictor or int4 or B != 1 else ncu_traffic(),
+                     "traffic": None if predictor or B != 1 else ncu_traffic("int4" if int4 else "bf16"),
                      "bytes_per_launch": gate_up_bytes,
                      "avg_launch_us": t_gate_up * 1e6},
         "e2e": e2e,
