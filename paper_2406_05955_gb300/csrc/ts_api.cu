@@ -10,6 +10,7 @@
 
 #include "ts_ffn.h"
 #include "ts_kernels.cuh"
+#include "ts_wide.h"
 
 using namespace tsffn;
 
@@ -45,7 +46,7 @@ ts_status device_info(DeviceInfo* di) {
         cudaSuccess)
         return TS_ERR_CUDA;
     if (prepare_gate_up(di->optin_smem) != cudaSuccess || prepare_down() != cudaSuccess ||
-        prepare_router() != cudaSuccess)
+        prepare_router() != cudaSuccess || prepare_wide() != cudaSuccess)
         return TS_ERR_CUDA;
     return TS_OK;
 }
@@ -108,6 +109,14 @@ struct ts_ffn {
     int last_n_rows = 0;
     int test_stall = 0;  // ts_ffn_set_test_stall
     int pass_max = kMaxPass;  // tokens per pass (kAccMaxTokens for INT4 rows)
+    // scratch of the wide kernels (batches of 9-64 tokens), when they apply
+    bool wide = false;
+    int wide_ks = 0;
+    float* w_gval = nullptr;            // [max_batch][m]
+    __nv_bfloat16* w_chi = nullptr;     // [m][64]
+    __nv_bfloat16* w_clo = nullptr;     // [m][64]
+    float* w_partial = nullptr;         // [ks][max_batch][d]
+    __nv_bfloat16* w_x = nullptr;       // [max_batch][d] normalised activations (stack)
 };
 
 struct ts_moe {
@@ -193,10 +202,27 @@ ts_status ts_ffn_create(ts_ffn** out, int d, int m, ts_dtype wdtype, const void*
     const size_t o_u = h->arena.take((size_t)h->nbytes);
     const size_t o_ug = h->arena.take((size_t)h->nbytes);
     const size_t o_s = h->arena.take(sizeof(unsigned));
+    h->wide = max_batch > kMaxPass && wide_supported(wdtype, d, m, max_batch);
+    size_t o_wg = 0, o_whi = 0, o_wlo = 0, o_wp = 0, o_wx = 0;
+    if (h->wide) {
+        h->wide_ks = wide_slices(d, dev.num_sms);
+        o_wg = h->arena.take((size_t)max_batch * m * sizeof(float));
+        o_whi = h->arena.take((size_t)m * 64 * sizeof(__nv_bfloat16));
+        o_wlo = h->arena.take((size_t)m * 64 * sizeof(__nv_bfloat16));
+        o_wp = h->arena.take((size_t)h->wide_ks * max_batch * d * sizeof(float));
+        o_wx = h->arena.take((size_t)max_batch * d * sizeof(__nv_bfloat16));
+    }
     st = alloc_arena(&h->arena);
     if (st != TS_OK) {
         delete h;
         return st;
+    }
+    if (h->wide) {
+        h->w_gval = h->arena.at<float>(o_wg);
+        h->w_chi = h->arena.at<__nv_bfloat16>(o_whi);
+        h->w_clo = h->arena.at<__nv_bfloat16>(o_wlo);
+        h->w_partial = h->arena.at<float>(o_wp);
+        h->w_x = h->arena.at<__nv_bfloat16>(o_wx);
     }
     h->s.cval = h->arena.at<float>(o_cval);
     h->s.gbits = h->arena.at<uint8_t>(o_g);
@@ -273,6 +299,34 @@ ts_status run_pass(ts_ffn* h, FfnLaunch a, int tok0, int nt, cudaStream_t stream
     return TS_OK;
 }
 
+// The whole batch in one wide pass (9-64 tokens, bf16 rows).
+bool use_wide(const ts_ffn* h, int batch) { return h->wide && wide_supported(h->dt, h->d, h->m, batch); }
+
+WideLaunch wide_launch(const ts_ffn* h, int batch, const int32_t* rows, int n_rows) {
+    WideLaunch L;
+    memset(&L, 0, sizeof L);
+    L.d = h->d;
+    L.m = h->m;
+    L.rows = rows;
+    L.n_rows = rows ? n_rows : h->m;
+    L.batch = batch;
+    L.wg = static_cast<const __nv_bfloat16*>(h->wg);
+    L.wu = static_cast<const __nv_bfloat16*>(h->wu);
+    L.wd = static_cast<const __nv_bfloat16*>(h->wd);
+    L.gval = h->w_gval;
+    L.c_hi = h->w_chi;
+    L.c_lo = h->w_clo;
+    L.partial = h->w_partial;
+    L.ks = h->wide_ks;
+    L.gbits = h->s.gbits;
+    L.bbits = h->s.bbits;
+    L.ubits = h->s.ubits;
+    L.ugbits = h->s.ugbits;
+    L.nbytes = h->nbytes;
+    L.status = h->s.status;
+    return L;
+}
+
 void remember(ts_ffn* h, int batch, const int32_t* rows, int n_rows) {
     h->last_batch = batch;
     h->last_rows = rows;
@@ -343,6 +397,14 @@ ts_status ts_ffn_forward(ts_ffn* h, const void* x, int batch, float* y, cudaStre
     if (!x || !y) return TS_ERR_INVALID_ARG;
     ts_status st = check_list(h, active_idx, n_active);
     if (st != TS_OK) return st;
+    if (use_wide(h, batch)) {
+        WideLaunch L = wide_launch(h, batch, active_idx, n_active);
+        L.x = static_cast<const __nv_bfloat16*>(x);
+        L.y = y;
+        st = cuda_status(launch_wide(L, stream, true));
+        if (st == TS_OK) remember(h, batch, active_idx, n_active);
+        return st;
+    }
     FfnLaunch a = ffn_launch(h, batch, active_idx, n_active);
     a.x = x;
     a.y = y;
@@ -396,6 +458,17 @@ ts_status ts_stack_forward(ts_ffn* const* layers, int n_layers, float* hres, int
         ts_ffn* h = layers[l];
         const int32_t* rows = active_idx ? active_idx[l] : nullptr;
         const int nr = rows ? n_active[l] : 0;
+        if (use_wide(h, batch)) {
+            WideLaunch L = wide_launch(h, batch, rows, nr);
+            L.x = h->w_x;
+            L.h = hres;
+            L.residual_out = 1;
+            ts_status st = cuda_status(launch_wide_norm(L, hres, h->w_x, stream, true));
+            if (st == TS_OK) st = cuda_status(launch_wide(L, stream, true));
+            if (st != TS_OK) return st;
+            remember(h, batch, rows, nr);
+            continue;
+        }
         FfnLaunch a = ffn_launch(h, batch, rows, nr);
         a.h = hres;
         a.norm_from_h = 1;

@@ -75,7 +75,7 @@ def test_ragged_shapes(ts, dtype, d, m, B):
     assert np.setxor1d(b, union_mask(ref, "both_mask")).size <= 2
 
 
-@pytest.mark.parametrize("B", [1, 4])
+@pytest.mark.parametrize("B", [1, 4, 16])
 def test_mistral_layer_full_size(ts, B):
     L = wl.ffn_layer(4096, 14336, activation=0.10, dtype=torch.bfloat16, seed=11)
     x = wl.tokens(B, 4096, dtype=torch.bfloat16, seed=12)
@@ -104,7 +104,7 @@ def test_activation_sweep(ts, act, B):
         assert len(b) == m
 
 
-@pytest.mark.parametrize("B", [1, 3, 8])
+@pytest.mark.parametrize("B", [1, 3, 8, 16])
 def test_predictor_lists(ts, B):
     d, m = 4096, 14336
     L = wl.ffn_layer(d, m, activation=0.10, dtype=torch.bfloat16, seed=21)

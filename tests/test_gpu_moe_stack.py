@@ -108,7 +108,7 @@ def test_moe_identical_experts_equal_single_ffn(ts):
     assert rel_l2(y_moe, y_one) <= 1e-5
 
 
-@pytest.mark.parametrize("B", [1, 3])
+@pytest.mark.parametrize("B", [1, 3, 16])
 @pytest.mark.parametrize("predictor", [False, True])
 def test_stack_teacher_forced(ts, B, predictor):
     d, m, n_layers = 1024, 3584, 4
@@ -133,8 +133,9 @@ def test_stack_teacher_forced(ts, B, predictor):
         h = (h.astype(np.float64) + ref["y"]).astype(np.float32)
 
 
-def test_stack_graph_equals_direct(ts):
-    d, m, n_layers, B = 1024, 3584, 3, 2
+@pytest.mark.parametrize("B", [2, 16])
+def test_stack_graph_equals_direct(ts, B):
+    d, m, n_layers = 1024, 3584, 3
     layers = [wl.ffn_layer(d, m, activation=0.10, dtype=torch.bfloat16, seed=wl.layer_seed(600, l))
               for l in range(n_layers)]
     dev = torch.device("cuda")
