@@ -62,6 +62,8 @@ def _load():
             lib.ts_oracle_ffn.restype = I
             lib.ts_oracle_ffn_w.argtypes = [I, I, I, I, P, I, P, P, P, P, I, P, P, P, P, P, I]
             lib.ts_oracle_ffn_w.restype = I
+            lib.ts_oracle_ffn_topk.argtypes = [I, I, I, I, P, I, P, P, P, I, P, P, P, P, I]
+            lib.ts_oracle_ffn_topk.restype = I
             lib.ts_oracle_router.argtypes = [I, I, I, I, P, P, I, P, P, P]
             lib.ts_oracle_router.restype = I
             lib.ts_oracle_rmsnorm.argtypes = [I, I, P, ctypes.c_double, I, P]
@@ -153,6 +155,37 @@ def ffn(x, w_gate, w_up, w_down, rows=None, threads: int = 0) -> dict:
     if rc != 0:
         raise ValueError("ts_oracle_ffn rejected its arguments (bad shape or row list)")
     return {"y": y, "g": g, "u": u, "gate_mask": gm, "both_mask": bm}
+
+
+def ffn_topk(x, w_gate, w_up, w_down, keep: int, threads: int = 0) -> dict:
+    """FFN with the top-k magnitude mask of Eq. 3 and Eq. 4: per token only the
+    ``keep`` neurons with the largest |Combined| (lower index first on a tie)
+    enter ``(Combined * Mask) W_down``. Same storage rules as ``ffn`` (no row
+    list). Returns float64 ``y [B][d]``, ``g``, ``u``, ``c`` ``[B][m]`` and uint8
+    ``sel [B][m]`` (the kept neurons)."""
+    x, w_gate, w_up, w_down = (as_array(a) for a in (x, w_gate, w_up, w_down))
+    if x.ndim == 1:
+        x = x[None, :]
+    B, d = x.shape
+    m = w_gate.shape[0]
+    dt, wdt = _dtype_of(x), _dtype_of(w_gate)
+    if dt == INT4:
+        raise ValueError("activations are fp32 or bf16")
+    for w in (w_gate, w_up, w_down):
+        if wdt == INT4:
+            if d % INT4_GROUP != 0 or w.shape != (m, int4_row_bytes(d)) or _dtype_of(w) != INT4:
+                raise ValueError("INT4 weights must be [m][d/2 + d/16] uint8, d a multiple of 32")
+        elif w.shape != (m, d) or _dtype_of(w) != dt:
+            raise ValueError("weights must be [m][d] in the activations' storage type")
+    g = np.zeros((B, m), np.float64)
+    u = np.zeros((B, m), np.float64)
+    sel = np.zeros((B, m), np.uint8)
+    y = np.zeros((B, d), np.float64)
+    rc = _load().ts_oracle_ffn_topk(d, m, B, dt, _ptr(x), wdt, _ptr(w_gate), _ptr(w_up), _ptr(w_down),
+                                    int(keep), _ptr(g), _ptr(u), _ptr(sel), _ptr(y), int(threads))
+    if rc != 0:
+        raise ValueError("ts_oracle_ffn_topk rejected its arguments")
+    return {"y": y, "g": g, "u": u, "c": np.maximum(g, 0) * np.maximum(u, 0), "sel": sel}
 
 
 def router(x, w_r, top_k: int = 2) -> dict:

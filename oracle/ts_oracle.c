@@ -212,6 +212,77 @@ int ts_oracle_ffn(int d, int m, int B, int dtype, const void* x, const void* w_g
 }
 
 /*
+ * Top-k magnitude mask (Eq. 3 and Eq. 4, Sec. 5): per token, Mask keeps the
+ * `keep` neurons with the largest |Combined| (Combined = max(0, g) max(0, u),
+ * Eq. 2), a lower neuron index winning a tie, and the output is
+ * (Combined * Mask) W_down.
+ *
+ *   x, w_gate, w_up, w_down, dtypes: as ts_oracle_ffn_w (no row list)
+ *   keep          neurons kept per token, 0 <= keep <= m
+ *   g, u [B][m]   out: the pre-activations (as ts_oracle_ffn_w)
+ *   sel  [B][m]   out: 1 iff the neuron is among the kept ones
+ *   y    [B][d]   out: sum over the kept neurons (ascending j) of
+ *                 Combined_j * W_down[j][:]
+ *
+ * The selection sorts all m neurons by (|Combined| descending, index
+ * ascending) and keeps the first `keep`. Returns 0, or -1 on invalid arguments.
+ */
+static const double* g_sort_key;
+static int by_magnitude_then_index(const void* pa, const void* pb) {
+    const int a = *(const int*)pa, b = *(const int*)pb;
+    const double ka = fabs(g_sort_key[a]), kb = fabs(g_sort_key[b]);
+    if (ka > kb) return -1;
+    if (ka < kb) return 1;
+    return a < b ? -1 : (a > b ? 1 : 0);
+}
+
+int ts_oracle_ffn_topk(int d, int m, int B, int dtype, const void* x, int wdtype, const void* w_gate,
+                       const void* w_up, const void* w_down, int keep, double* g, double* u, uint8_t* sel,
+                       double* y, int n_threads) {
+    if (keep < 0 || keep > m || B < 0) return -1;
+    uint8_t* gm = (uint8_t*)malloc((size_t)B * (size_t)m + 1);
+    uint8_t* bm = (uint8_t*)malloc((size_t)B * (size_t)m + 1);
+    double* c = (double*)malloc(sizeof(double) * (size_t)m);
+    int* order = (int*)malloc(sizeof(int) * (size_t)m);
+    if (!gm || !bm || !c || !order) {
+        free(gm);
+        free(bm);
+        free(c);
+        free(order);
+        return -1;
+    }
+    /* g and u of every neuron (the plain FFN's y is overwritten below) */
+    int rc = ts_oracle_ffn_w(d, m, B, dtype, x, wdtype, w_gate, w_up, w_down, NULL, 0, g, u, gm, bm, y,
+                             n_threads);
+    for (int b = 0; rc == 0 && b < B; ++b) {
+        const double* gb = g + (size_t)b * (size_t)m;
+        const double* ub = u + (size_t)b * (size_t)m;
+        uint8_t* sb = sel + (size_t)b * (size_t)m;
+        for (int j = 0; j < m; ++j) {
+            c[j] = relu(gb[j]) * relu(ub[j]); /* Eq. 2 */
+            order[j] = j;
+            sb[j] = 0;
+        }
+        g_sort_key = c;
+        qsort(order, (size_t)m, sizeof(int), by_magnitude_then_index);
+        for (int q = 0; q < keep; ++q) sb[order[q]] = 1; /* Eq. 3 */
+        /* Eq. 4: (Combined * Mask) W_down, j ascending */
+        double* yb = y + (size_t)b * (size_t)d;
+        for (int i = 0; i < d; ++i) yb[i] = 0.0;
+        for (int j = 0; j < m; ++j) {
+            if (!sb[j]) continue;
+#pragma omp parallel for schedule(static)
+            for (int i = 0; i < d; ++i) yb[i] += c[j] * welem(w_down, wdtype, d, j, i);
+        }
+    }
+    free(gm);
+    free(bm);
+    free(c);
+    free(order);
+    return rc;
+}
+
+/*
  * Router of a top-k MoE layer (Sec. 4; Mixtral routes each token to 2 of 8
  * experts, Sec. 6.2): logits r_e = sum_i W_r[e][i] x_i; the k experts with
  * the largest logits are chosen, a lower expert index winning a tie; their
