@@ -446,6 +446,78 @@ def _clocked_time(graph, stream, steps, dist):
     return dist.max(elapsed), clocks.stop()
 
 
+class _Calls:
+    """A list of launches that time_graph can replay like a graph."""
+
+    def __init__(self, fn):
+        self.fn = fn
+
+    def launch(self, stream):
+        self.fn(stream)
+
+
+def run_topk(args, dist: Dist) -> dict:
+    """Top-k magnitude mask (Eq. 3-4) on 32 full-size layers at batch 1: per
+    layer one ts_ffn_forward_topk on the token's normalised activations
+    (the same x for every layer: the mask, not the stack glue, is measured)."""
+    import paper_2406_05955_gb300 as ts
+    from paper_2406_05955_gb300 import workload as wl
+
+    name = "mistral7b-ffn-topk5-b1"
+    cfg = wl.WORKLOADS[name]
+    dev = torch.device("cuda", dist.local)
+    torch.cuda.set_device(dev)
+    d, m, B, keep = cfg["d"], cfg["m"], cfg["batch"], cfg["keep"]
+    n_layers = args.layers or cfg["layers"]
+    layers = [wl.ffn_layer(d, m, activation=cfg["activation"], dtype=torch.bfloat16,
+                           seed=wl.layer_seed(cfg["seed"], l), device=dev) for l in range(n_layers)]
+    ffns = [ts.Ffn(L.w_gate, L.w_up, L.w_down, max_batch=B) for L in layers]
+    x = wl.tokens(B, d, dtype=torch.bfloat16, seed=cfg["seed"] + 7, device=dev)
+    y = torch.empty(B, d, dtype=torch.float32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step_topk(s):
+        for f in ffns:
+            f.forward_topk(x, keep, y=y, stream=s)
+
+    def step_plain(s):
+        for f in ffns:
+            f.forward(x, y=y, stream=s)
+
+    calls = _Calls(step_topk)
+    for _ in range(args.warmup):
+        calls.launch(stream)
+    torch.cuda.synchronize()
+    t_max, clk = _clocked_time(calls, stream, args.steps, dist)
+    value = whole_job_value(B, args.steps, dist.world, t_max)
+    kept = statistics.mean(len(f.get_active(0)[1]) for f in ffns)
+    plain = _Calls(step_plain)
+    for _ in range(args.warmup):
+        plain.launch(stream)
+    torch.cuda.synchronize()
+    t_plain = time_graph(plain, stream, args.steps)
+    step_s = t_max / args.steps
+    nb = needed_bytes_stack(ffns, None)  # gate rows + gate-active up rows + kept down rows
+    peaks = load_peaks()
+    return {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": name, "d": d, "m": m, "layers": n_layers, "batch": B, "keep": keep,
+                   "activation": cfg["activation"],
+                   "l2": "no flush: the 11.3 GB of weights streamed per step exceed the 129 MB L2",
+                   "parallelism": f"replicas x{dist.world}"},
+        "kept_per_layer": kept,
+        "needed_bytes_roofline": {
+            "bytes_per_token": (nb["gate_up"] + nb["down"]) / B,
+            "achieved_gbs": (nb["gate_up"] + nb["down"]) / step_s / 1e9,
+            "frac_of_measured": (nb["gate_up"] + nb["down"]) / step_s / 1e9 / peaks["hbm_gbs"]},
+        "plain_forward_same_layers": {"value": B * args.steps / t_plain, "unit": UNIT},
+        "gpu_launches": 4 * n_layers * args.steps,
+        "clocks": clk,
+    }
+
+
 def run_moe(args, dist: Dist) -> dict:
     """32-layer Mixtral-shaped MoE stack (router + top-2 of 8 sparse experts per layer)."""
     import paper_2406_05955_gb300 as ts
@@ -610,7 +682,8 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["stack", "predictor", "moe", "sweep", "int4", "moe-int4"], default="stack")
+    ap.add_argument("--workload", choices=["stack", "predictor", "moe", "sweep", "int4", "moe-int4", "topk"],
+                    default="stack")
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--layers", type=int, default=0,
                     help="fewer layers than the workload's 32 (profiling cases only; not a bench line)")
@@ -635,6 +708,8 @@ def main():
                 res = run_moe(args, dist)
             elif args.workload == "sweep":
                 res = run_sweep(args, dist)
+            elif args.workload == "topk":
+                res = run_topk(args, dist)
             else:
                 res = run_ours(args, dist)
         if res is not None and dist.rank == 0:

@@ -103,6 +103,21 @@ ts_status ts_ffn_forward(ts_ffn* h, const void* x, int batch, float* y, cudaStre
                          const int32_t* active_idx, int n_active);
 
 /*
+ * y = (Combined(x) * Mask(x)) W_down with the top-k magnitude mask of Eq. 3
+ * and Eq. 4 (Sec. 5): per token, Mask keeps the `keep` neurons with the
+ * largest |Combined| = max(0, g) max(0, u) (Eq. 2), a lower neuron index
+ * winning a tie; the others contribute 0.
+ *   x, batch, y, stream   as ts_ffn_forward (no predictor list)
+ *   keep                  0 <= keep <= m; keep >= the number of dReLU-active
+ *                         neurons gives exactly ts_ffn_forward's result
+ * The per-token both-active sets that ts_ffn_get_active reports afterwards
+ * are the kept active neurons. The selection compares the fp32 c values.
+ * Errors: TS_ERR_INVALID_ARG for a bad keep or batch, TS_ERR_UNSUPPORTED for
+ * INT4 rows.
+ */
+ts_status ts_ffn_forward_topk(ts_ffn* h, const void* x, int batch, float* y, cudaStream_t stream, int keep);
+
+/*
  * First step alone: gate GEMV + ReLU + compaction, then the gathered up
  * projection over gate-active rows + dReLU product + second compaction
  * (into the handle's scratch). Arguments as ts_ffn_forward. For batch > 8

@@ -36,6 +36,7 @@ SIGNATURES = {
     "ts_ffn_create": (I, [PP, I, I, I, P, P, P, I]),
     "ts_ffn_destroy": (None, [P]),
     "ts_ffn_forward": (I, [P, P, I, P, P, P, I]),
+    "ts_ffn_forward_topk": (I, [P, P, I, P, P, I]),
     "ts_ffn_gate_up": (I, [P, P, I, P, P, I]),
     "ts_ffn_down": (I, [P, I, P, P]),
     "ts_stack_forward": (I, [P, I, P, I, P, P, P]),
@@ -188,6 +189,16 @@ class Ffn:
         return y
 
     __call__ = forward
+
+    def forward_topk(self, x, keep: int, y=None, stream=None) -> torch.Tensor:
+        """``ts_ffn_forward_topk``: the top-k magnitude mask of Eq. 3-4."""
+        x = self._x(x)
+        if y is None:
+            y = torch.empty(x.shape[0], self.d, dtype=torch.float32, device=x.device)
+        _dev(y, "y")
+        _check(lib().ts_ffn_forward_topk(self.handle, x.data_ptr(), x.shape[0], y.data_ptr(),
+                                         _stream(stream), int(keep)), "ts_ffn_forward_topk")
+        return y
 
     def gate_up(self, x, active_idx=None, stream=None) -> None:
         x = self._x(x)

@@ -416,6 +416,31 @@ ts_status ts_ffn_forward(ts_ffn* h, const void* x, int batch, float* y, cudaStre
     return TS_OK;
 }
 
+ts_status ts_ffn_forward_topk(ts_ffn* h, const void* x, int batch, float* y, cudaStream_t stream, int keep) {
+    if (!h || batch < 0 || batch > h->max_batch || keep < 0 || keep > h->m) return TS_ERR_INVALID_ARG;
+    if (h->dt == TS_INT4) return TS_ERR_UNSUPPORTED;
+    if (batch == 0) return TS_OK;
+    if (!x || !y) return TS_ERR_INVALID_ARG;
+    FfnLaunch a = ffn_launch(h, batch, nullptr, 0);
+    a.x = x;
+    a.y = y;
+    for (int t0 = 0; t0 < batch; t0 += kMaxPass) {
+        // passes of at least 4 tokens: the down projection runs after the mask
+        const int nt = std::min(kMaxPass, batch - t0);
+        const int w = std::max(4, pow2_tokens(nt));
+        a.tok0 = t0;
+        a.nt = nt;
+        a.bits_tok_base = t0;
+        a.partial_ctas = h->grid[w];
+        ts_status st = cuda_status(launch_gate_up(a, h->dt, w, h->grid[w], stream, true));
+        if (st == TS_OK) st = cuda_status(launch_topk(a, keep, stream));
+        if (st == TS_OK) st = cuda_status(launch_down(a, h->dt, w, stream, true));
+        if (st != TS_OK) return st;
+    }
+    remember(h, batch, nullptr, 0);
+    return TS_OK;
+}
+
 ts_status ts_ffn_gate_up(ts_ffn* h, const void* x, int batch, cudaStream_t stream,
                          const int32_t* active_idx, int n_active) {
     if (!h || batch < 0 || batch > h->max_batch) return TS_ERR_INVALID_ARG;

@@ -334,6 +334,8 @@ __device__ __forceinline__ void block_rmsnorm(const float* __restrict__ h, int d
 namespace tsffn {
 cudaError_t launch_gate_up(const FfnLaunch& a, int wdtype, int pass_tokens, int grid,
                            cudaStream_t stream, bool pdl);
+// Top-k magnitude mask (Eq. 3-4) on a pass's c values and both-active bitmaps.
+cudaError_t launch_topk(const FfnLaunch& a, int keep, cudaStream_t stream);
 cudaError_t launch_down(const FfnLaunch& a, int wdtype, int pass_tokens, cudaStream_t stream,
                         bool pdl);
 // Sum of the gate+up CTAs' partial down projections (passes of <= kAccMaxTokens).

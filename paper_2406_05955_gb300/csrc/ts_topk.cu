@@ -1,0 +1,143 @@
+// ts_topk.cu -- the top-k magnitude mask of Eq. 3-4 between the gate+up and
+// the down launches of a pass: per token, only the `keep` neurons with the
+// largest |Combined| (Combined = max(0, g) max(0, u), Eq. 2; a lower neuron
+// index wins a tie) keep their c; the down projection then sums
+// (Combined * Mask) W_down. Candidates are the token's both-active rows (every
+// other row has Combined = 0 and adds nothing whether kept or not).
+#include "ts_kernels.cuh"
+
+namespace tsffn {
+namespace {
+
+constexpr int kSelThreads = 1024;
+
+// One CTA per token of the pass. c > 0 at a both-active row, so the fp32 bit
+// pattern orders the candidates; an MSB-first radix select (four 8-bit
+// digits) finds the keep-th largest key T, then the rows with key > T and the
+// first rows (ascending) with key == T are kept. Threads own contiguous byte
+// ranges of the bitmap, so a block prefix over the threads is row order.
+__global__ void __launch_bounds__(kSelThreads) k_topk_select(const FfnLaunch a, int keep) {
+    __shared__ unsigned hist[256];
+    __shared__ int s_part[kSelThreads];
+    __shared__ unsigned s_prefix, s_mask;
+    __shared__ int s_remaining, s_total;
+    pdl_wait();
+    pdl_launch_dependents();
+    const int k = blockIdx.x;  // batch slot of the pass
+    const int tid = threadIdx.x;
+    float* cv = a.cval + (size_t)k * a.cval_tok_stride;
+    uint8_t* bb = a.bbits + (size_t)(a.bits_tok_base + k) * a.nbytes;
+    const int n_bytes = (a.n_rows + 7) / 8;
+    const int per = (n_bytes + kSelThreads - 1) / kSelThreads;
+    const int b0 = min(tid * per, n_bytes), b1 = min(b0 + per, n_bytes);
+    auto key_of = [&](int p) { return __float_as_uint(cv[p]); };
+
+    // candidates
+    int cnt = 0;
+    for (int b = b0; b < b1; ++b) cnt += __popc((unsigned)bb[b]);
+    s_part[tid] = cnt;
+    __syncthreads();
+    if (tid == 0) {
+        int t = 0;
+        for (int i = 0; i < kSelThreads; ++i) t += s_part[i];
+        s_total = t;
+        s_prefix = 0u;
+        s_mask = 0u;
+        s_remaining = keep;
+    }
+    __syncthreads();
+    if (keep >= s_total) return;  // every candidate is kept
+
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
+        __syncthreads();
+        const unsigned prefix = s_prefix, mask = s_mask;
+        for (int b = b0; b < b1; ++b)
+            for (unsigned bits = bb[b]; bits; bits &= bits - 1u) {
+                const int p = b * 8 + __ffs(bits) - 1;
+                const unsigned key = key_of(p);
+                if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+            }
+        __syncthreads();
+        if (tid == 0) {
+            // the digit of the keep-th largest key among those with the prefix
+            int remaining = s_remaining;
+            int dg = 255;
+            for (; dg > 0; --dg) {
+                if ((int)hist[dg] >= remaining) break;
+                remaining -= (int)hist[dg];
+            }
+            s_prefix = prefix | ((unsigned)dg << shift);
+            s_mask = mask | (255u << shift);
+            s_remaining = remaining;  // how many keys equal to the final prefix are kept, at the end
+        }
+        __syncthreads();
+    }
+    const unsigned T = s_prefix;
+    const int need_eq = s_remaining;
+    // rank of each key == T in row order
+    int eq = 0;
+    for (int b = b0; b < b1; ++b)
+        for (unsigned bits = bb[b]; bits; bits &= bits - 1u) eq += key_of(b * 8 + __ffs(bits) - 1) == T;
+    s_part[tid] = eq;
+    __syncthreads();
+    if (tid == 0) {
+        int run = 0;
+        for (int i = 0; i < kSelThreads; ++i) {
+            const int v = s_part[i];
+            s_part[i] = run;
+            run += v;
+        }
+    }
+    __syncthreads();
+    int rank = s_part[tid];
+    for (int b = b0; b < b1; ++b) {
+        unsigned kept = 0u;
+        for (unsigned bits = bb[b]; bits; bits &= bits - 1u) {
+            const int r = __ffs(bits) - 1;
+            const int p = b * 8 + r;
+            const unsigned key = key_of(p);
+            bool keep_it = key > T;
+            if (key == T) keep_it = rank++ < need_eq;
+            if (keep_it)
+                kept |= 1u << r;
+            else
+                cv[p] = 0.0f;  // the down projection multiplies by c
+        }
+        bb[b] = (uint8_t)kept;
+    }
+}
+
+// The pass's union both-active bytes from the masked per-token bytes.
+__global__ void __launch_bounds__(256) k_topk_union(const FfnLaunch a) {
+    pdl_wait();
+    pdl_launch_dependents();
+    const int n_bytes = (a.n_rows + 7) / 8;
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b >= n_bytes) return;
+    unsigned u = 0u;
+    for (int k = 0; k < a.nt; ++k) u |= a.bbits[(size_t)(a.bits_tok_base + k) * a.nbytes + b];
+    a.ubits[b] = (uint8_t)u;
+}
+
+}  // namespace
+
+cudaError_t launch_topk(const FfnLaunch& a, int keep, cudaStream_t stream) {
+    cudaLaunchConfig_t lc = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    lc.stream = stream;
+    lc.gridDim = dim3(a.nt);
+    lc.blockDim = dim3(kSelThreads);
+    cudaError_t e = cudaLaunchKernelEx(&lc, k_topk_select, a, keep);
+    if (e != cudaSuccess) return e;
+    const int n_bytes = (a.n_rows + 7) / 8;
+    lc.gridDim = dim3((n_bytes + 255) / 256);
+    lc.blockDim = dim3(256);
+    return cudaLaunchKernelEx(&lc, k_topk_union, a);
+}
+
+}  // namespace tsffn

@@ -210,6 +210,10 @@ WORKLOADS = {
         d=MISTRAL_D, m=MISTRAL_M, dtype="int4", experts=8, top_k=2, batches=(1,), layers=N_LAYERS,
         activation=0.20, seed=3000,
         desc="the Mixtral-shaped MoE stack with INT4 experts (the paper's Mixtral-47B-INT4 setting)"),
+    "mistral7b-ffn-topk5-b1": dict(
+        d=MISTRAL_D, m=MISTRAL_M, dtype="bf16", batch=1, layers=N_LAYERS, activation=0.10, keep=717,
+        seed=1000,
+        desc="top-k magnitude mask (Eq. 3-4) keeping 717 of 14336 neurons (5%) per token, 32 layers at ~10% dReLU activity"),
     "mistral7b-ffn-stack-bf16-predictor": dict(
         d=MISTRAL_D, m=MISTRAL_M, dtype="bf16", batch=1, layers=N_LAYERS, activation=0.10,
         list_len=1434, zipf_s=1.1, seed=1000,
