@@ -64,6 +64,8 @@ def _load():
             lib.ts_oracle_ffn_w.restype = I
             lib.ts_oracle_ffn_topk.argtypes = [I, I, I, I, P, I, P, P, P, I, P, P, P, P, I]
             lib.ts_oracle_ffn_topk.restype = I
+            lib.ts_oracle_predict.argtypes = [I, I, I, I, I, P, P, P, I, P, P]
+            lib.ts_oracle_predict.restype = I
             lib.ts_oracle_router.argtypes = [I, I, I, I, P, P, I, P, P, P]
             lib.ts_oracle_router.restype = I
             lib.ts_oracle_rmsnorm.argtypes = [I, I, P, ctypes.c_double, I, P]
@@ -186,6 +188,28 @@ def ffn_topk(x, w_gate, w_up, w_down, keep: int, threads: int = 0) -> dict:
     if rc != 0:
         raise ValueError("ts_oracle_ffn_topk rejected its arguments")
     return {"y": y, "g": g, "u": u, "c": np.maximum(g, 0) * np.maximum(u, 0), "sel": sel}
+
+
+def predict(x, w1, w2, K: int) -> dict:
+    """Activation predictor (a two-layer ReLU MLP, the reading of Sec. 7's
+    predictor): ``s = W2 max(0, W1 x)`` per token; the list is the K neurons
+    with the largest max-over-tokens score (lower index first on a tie), in
+    ascending order. Returns float64 ``scores [B][m]`` and int32 ``list [K]``."""
+    x, w1, w2 = (as_array(a) for a in (x, w1, w2))
+    if x.ndim == 1:
+        x = x[None, :]
+    B, d = x.shape
+    r = w1.shape[0]
+    m = w2.shape[0]
+    dt = _dtype_of(x)
+    if dt == INT4 or w1.shape != (r, d) or w2.shape != (m, r) or _dtype_of(w1) != dt or _dtype_of(w2) != dt:
+        raise ValueError("predictor weights are W1 [r][d] and W2 [m][r] in the activations' storage type")
+    scores = np.zeros((B, m), np.float64)
+    lst = np.zeros(max(K, 1), np.int32)
+    rc = _load().ts_oracle_predict(d, r, m, B, dt, _ptr(x), _ptr(w1), _ptr(w2), int(K), _ptr(scores), _ptr(lst))
+    if rc != 0:
+        raise ValueError("ts_oracle_predict rejected its arguments")
+    return {"scores": scores, "list": lst[:K]}
 
 
 def router(x, w_r, top_k: int = 2) -> dict:

@@ -236,6 +236,15 @@ static int by_magnitude_then_index(const void* pa, const void* pb) {
     return a < b ? -1 : (a > b ? 1 : 0);
 }
 
+static const double* g_sort_key_signed;
+static int by_value_then_index(const void* pa, const void* pb) {
+    const int a = *(const int*)pa, b = *(const int*)pb;
+    const double ka = g_sort_key_signed[a], kb = g_sort_key_signed[b];
+    if (ka > kb) return -1;
+    if (ka < kb) return 1;
+    return a < b ? -1 : (a > b ? 1 : 0);
+}
+
 int ts_oracle_ffn_topk(int d, int m, int B, int dtype, const void* x, int wdtype, const void* w_gate,
                        const void* w_up, const void* w_down, int keep, double* g, double* u, uint8_t* sel,
                        double* y, int n_threads) {
@@ -280,6 +289,72 @@ int ts_oracle_ffn_topk(int d, int m, int B, int dtype, const void* x, int wdtype
     free(c);
     free(order);
     return rc;
+}
+
+/*
+ * Activation predictor (Sec. 7 names a predictor per FFN block without its
+ * architecture; reading: a two-layer ReLU MLP of rank r that outputs, for a
+ * batch, the list of the K neurons it rates most likely to be active):
+ *   h_t   = max(0, W1 x_t)                 W1 [r][d], h_t [r]
+ *   s_t,j = sum_i W2[j][i] h_t,i           W2 [m][r]
+ *   key_j = max over the batch's tokens of s_t,j
+ * The K neurons with the largest key (a lower index winning a tie) are the
+ * list, in ascending neuron order.
+ *
+ *   x [B][d] (dtype), w1 [r][d], w2 [m][r] (wdtype = dtype); K: 0 <= K <= m
+ *   scores [B][m] out: s;  list [K] out: ascending neuron ids
+ * Returns 0, or -1 on invalid arguments.
+ */
+int ts_oracle_predict(int d, int r, int m, int B, int dtype, const void* x, const void* w1, const void* w2,
+                      int K, double* scores, int32_t* list) {
+    if (d <= 0 || r <= 0 || m <= 0 || B <= 0 || K < 0 || K > m) return -1;
+    if (dtype != ORACLE_F32 && dtype != ORACLE_BF16) return -1;
+    double* h = (double*)malloc(sizeof(double) * (size_t)r);
+    double* key = (double*)malloc(sizeof(double) * (size_t)m);
+    int* order = (int*)malloc(sizeof(int) * (size_t)m);
+    uint8_t* pick = (uint8_t*)calloc((size_t)m, 1);
+    if (!h || !key || !order || !pick) {
+        free(h);
+        free(key);
+        free(order);
+        free(pick);
+        return -1;
+    }
+    for (int b = 0; b < B; ++b) {
+        for (int i = 0; i < r; ++i) {
+            double v = 0.0;
+            for (int k = 0; k < d; ++k)
+                v += elem(w1, dtype, (size_t)i * (size_t)d + (size_t)k) * elem(x, dtype, (size_t)b * (size_t)d + (size_t)k);
+            h[i] = relu(v);
+        }
+        double* sb = scores + (size_t)b * (size_t)m;
+#pragma omp parallel for schedule(static)
+        for (int j = 0; j < m; ++j) {
+            double v = 0.0;
+            for (int i = 0; i < r; ++i) v += elem(w2, dtype, (size_t)j * (size_t)r + (size_t)i) * h[i];
+            sb[j] = v;
+        }
+    }
+    for (int j = 0; j < m; ++j) {
+        double kj = scores[j];
+        for (int b = 1; b < B; ++b) {
+            const double v = scores[(size_t)b * (size_t)m + (size_t)j];
+            if (v > kj) kj = v;
+        }
+        key[j] = kj;
+        order[j] = j;
+    }
+    g_sort_key_signed = key;
+    qsort(order, (size_t)m, sizeof(int), by_value_then_index);
+    for (int q = 0; q < K; ++q) pick[order[q]] = 1;
+    int n = 0;
+    for (int j = 0; j < m; ++j)
+        if (pick[j]) list[n++] = j;
+    free(h);
+    free(key);
+    free(order);
+    free(pick);
+    return 0;
 }
 
 /*

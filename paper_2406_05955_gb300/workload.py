@@ -145,6 +145,28 @@ def ffn_layer_int4(d: int, m: int, *, activation: float = 0.10, mu: float | None
                         L.offsets, d)
 
 
+@dataclass
+class Predictor:
+    w1: torch.Tensor  # [r][d]
+    w2: torch.Tensor  # [m][r]
+
+
+def predictor_weights(d: int, r: int, m: int, offsets: torch.Tensor, *, dtype=torch.bfloat16, seed: int = 0,
+                      device="cpu") -> Predictor:
+    """Synthetic weights of the rank-r activation predictor (a two-layer ReLU
+    MLP): W1 ~ N(0, 1/d) with its last row picking the bias channel x[d-1] = 1
+    (so that hidden unit is constantly 1), W2 ~ N(0, 1/r) with its last column
+    holding the layer's per-neuron offsets b_j, which favours the layer's hot
+    neurons. Trained weights do not exist here; these only have the shapes."""
+    g = _gen(seed, device)
+    w1 = torch.randn(r, d, generator=g, device=device) / math.sqrt(d)
+    w1[r - 1] = 0.0
+    w1[r - 1, d - 1] = 1.0
+    w2 = torch.randn(m, r, generator=g, device=device) / math.sqrt(r)
+    w2[:, r - 1] = offsets.to(device=device, dtype=torch.float32)
+    return Predictor(w1.to(dtype).contiguous(), w2.to(dtype).contiguous())
+
+
 def tokens(B: int, d: int, *, dtype=torch.bfloat16, seed: int = 0, device="cpu") -> torch.Tensor:
     """Token activations ``[B][d]``: N(0,1) entries with the bias channel ``x[:, d-1] = 1``."""
     x = torch.randn(B, d, generator=_gen(seed, device), device=device)
