@@ -518,6 +518,84 @@ def run_topk(args, dist: Dist) -> dict:
     }
 
 
+def run_prednet(args, dist: Dist) -> dict:
+    """Predictor network + predictor mode on the 32-layer Mistral-shaped stack
+    at batch 1: per layer, a rank-512 two-layer ReLU MLP scores the 14336
+    neurons from rmsnorm(h), the 1434 best form the list, and the FFN runs
+    over the listed rows only; the whole step is one CUDA graph."""
+    import paper_2406_05955_gb300 as ts
+    from paper_2406_05955_gb300 import workload as wl
+
+    name = "mistral7b-ffn-stack-bf16-b1-prednet"
+    cfg = dict(wl.WORKLOADS[name])
+    dev = torch.device("cuda", dist.local)
+    torch.cuda.set_device(dev)
+    d, m, r, K, B = cfg["d"], cfg["m"], cfg["rank"], cfg["k"], cfg["batch"]
+    n_layers = args.layers or cfg["layers"]
+    layers, ffns, preds, pw = [], [], [], []
+    for l in range(n_layers):
+        L = wl.ffn_layer(d, m, activation=cfg["activation"], dtype=torch.bfloat16,
+                         seed=wl.layer_seed(cfg["seed"], l), device=dev)
+        P = wl.predictor_weights(d, r, m, L.offsets, dtype=torch.bfloat16,
+                                 seed=wl.layer_seed(cfg["seed"], l) + 11, device=dev)
+        layers.append(L)
+        pw.append(P)
+        ffns.append(ts.Ffn(L.w_gate, L.w_up, L.w_down, max_batch=B))
+        preds.append(ts.Predictor(P.w1, P.w2, max_batch=B))
+    lists = [torch.empty(K, dtype=torch.int32, device=dev) for _ in range(n_layers)]
+    h0 = wl.residual(B, d, seed=cfg["seed"] - 1, device=dev)
+    h = h0.clone()
+    stream = torch.cuda.Stream(device=dev)
+    graph = ts.Graph.stack_predicted(ffns, preds, h, [K] * n_layers, lists)
+    for _ in range(args.warmup):
+        graph.launch(stream)
+    torch.cuda.synchronize()
+    t_max, clk = _clocked_time(graph, stream, args.steps, dist)
+    value = whole_job_value(B, args.steps, dist.world, t_max)
+    step_s = t_max / args.steps
+    # algorithmic bytes: both predictor matrices, then the FFN over the lists
+    nb = needed_bytes_stack(ffns, lists)
+    pred_bytes = n_layers * (r * d + m * r) * 2
+    total = nb["gate_up"] + nb["down"] + pred_bytes
+    peaks = load_peaks()
+
+    # the prediction alone (3 launches per layer), CUDA events on its stream
+    x = wl.tokens(B, d, dtype=torch.bfloat16, seed=cfg["seed"] + 5, device=dev)
+    for p_, buf in zip(preds, lists):
+        p_.predict(x, K, out=buf, stream=stream)
+    torch.cuda.synchronize()
+    s_ev, e_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 5
+    s_ev.record(stream)
+    for _ in range(reps):
+        for p_, buf in zip(preds, lists):
+            p_.predict(x, K, out=buf, stream=stream)
+    e_ev.record(stream)
+    e_ev.synchronize()
+    t_pred = s_ev.elapsed_time(e_ev) / 1e3 / (reps * n_layers)
+    pred_layer_bytes = (r * d + m * r) * 2
+    res = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": name, "d": d, "m": m, "rank": r, "k": K, "layers": n_layers, "batch": B,
+                   "activation": cfg["activation"],
+                   "l2": "no flush: the 12 GB of FFN and predictor weights touched per step exceed the 129 MB L2",
+                   "parallelism": f"replicas x{dist.world}"},
+        "needed_bytes_roofline": {
+            "bytes_per_token": total / B, "predictor_bytes_per_token": pred_bytes / B,
+            "achieved_gbs": total / step_s / 1e9,
+            "frac_of_measured": total / step_s / 1e9 / peaks["hbm_gbs"]},
+        "prediction_only": {"us_per_layer": t_pred * 1e6,
+                            "achieved_gbs": pred_layer_bytes / t_pred / 1e9,
+                            "frac_of_measured": pred_layer_bytes / t_pred / 1e9 / peaks["hbm_gbs"]},
+        # per layer: hidden, score, select, gate+up, down reduction
+        "gpu_launches": 5 * n_layers * args.steps,
+        "clocks": clk,
+    }
+    return res
+
+
 def run_moe(args, dist: Dist) -> dict:
     """32-layer Mixtral-shaped MoE stack (router + top-2 of 8 sparse experts per layer)."""
     import paper_2406_05955_gb300 as ts
@@ -682,7 +760,8 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["stack", "predictor", "moe", "sweep", "int4", "moe-int4", "topk"],
+    ap.add_argument("--workload", choices=["stack", "predictor", "moe", "sweep", "int4", "moe-int4", "topk",
+                                           "prednet"],
                     default="stack")
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--layers", type=int, default=0,
@@ -710,6 +789,8 @@ def main():
                 res = run_sweep(args, dist)
             elif args.workload == "topk":
                 res = run_topk(args, dist)
+            elif args.workload == "prednet":
+                res = run_prednet(args, dist)
             else:
                 res = run_ours(args, dist)
         if res is not None and dist.rank == 0:

@@ -63,6 +63,7 @@ typedef enum { TS_F32 = 0, TS_BF16 = 1, TS_INT4 = 2 } ts_dtype;
 typedef struct ts_ffn ts_ffn;     /* one dReLU FFN (one layer or one expert) */
 typedef struct ts_moe ts_moe;     /* one top-k MoE layer over ts_ffn experts */
 typedef struct ts_graph ts_graph; /* a captured multi-layer forward          */
+typedef struct ts_predictor ts_predictor; /* one layer's activation predictor */
 
 /* Human-readable name of a status code (static string, never NULL). */
 const char* ts_status_str(ts_status s);
@@ -236,6 +237,50 @@ ts_status ts_moe_get_active(ts_moe* h, cudaStream_t stream, int expert, int toke
 ts_status ts_moe_get_error(ts_moe* h, cudaStream_t stream);
 
 /*
+ * Activation predictor of one FFN layer (Sec. 7: a predictor per FFN block,
+ * per expert for MoE; the paper gives no architecture, so this is a reading):
+ * a two-layer ReLU MLP over the layer's input x,
+ *     hid = max(0, W1 x),   s = W2 hid      (s[j]: score of neuron j),
+ * and a batch's list is the K neurons with the largest key
+ * key[j] = max over the batch's tokens of s[t][j], a lower neuron id winning
+ * a tie, emitted in ascending id order -- the input of the predictor-driven
+ * mode of ts_ffn_forward / ts_stack_forward.
+ *   d, r, m    input width, hidden width, neurons; d and r multiples of 256
+ *              (bf16) or 128 (fp32), r / that multiple one of 1, 2, 4, 8
+ *   dtype      TS_BF16 or TS_F32: the type of W1, W2 and x
+ *   w1, w2     device [r][d] and [m][r], row-major (borrowed, 16-byte aligned)
+ *   max_batch  largest batch of a prediction, 1..8
+ * Scores accumulate in fp32. Returns TS_ERR_UNSUPPORTED for sizes without a
+ * kernel, TS_ERR_OOM if scratch cannot be allocated.
+ */
+ts_status ts_predictor_create(ts_predictor** out, int d, int r, int m, ts_dtype dtype, const void* w1,
+                              const void* w2, int max_batch);
+void ts_predictor_destroy(ts_predictor* p);
+
+/*
+ * list[0..K) = the predicted neurons for the batch x [batch][d] (device,
+ * predictor dtype), ascending; `list` is a caller-owned device buffer of at
+ * least K int32. scores: NULL, or a device [batch][m] fp32 buffer that
+ * receives s. batch == 0 or K == 0 is a no-op. 0 <= K <= m, else
+ * TS_ERR_INVALID_ARG. Asynchronous on `stream`.
+ */
+ts_status ts_predict(ts_predictor* p, const void* x, int batch, int K, int32_t* list, float* scores,
+                     cudaStream_t stream);
+
+/*
+ * ts_stack_forward with a predictor per layer: for each layer l,
+ *     x = round_wdtype(h / sqrt(mean(h^2) + 1e-5)),  x[d-1] = 1,
+ *     lists[l][0..K[l]) = ts_predict(preds[l], x, K[l]),
+ *     h = h + FFN_l(x) over the listed neurons only (predictor-driven mode).
+ * preds[l] must match layer l's d, m and activation dtype (bf16 for INT4
+ * layers). lists[l]: caller-owned device buffers of K[l] int32 that keep the
+ * lists for inspection. K[l] == 0 leaves h unchanged for that layer.
+ */
+ts_status ts_stack_forward_predicted(ts_ffn* const* layers, ts_predictor* const* preds, int n_layers,
+                                     float* h, int batch, const int* K, int32_t* const* lists,
+                                     cudaStream_t stream);
+
+/*
  * Capture a whole multi-layer forward once as a CUDA graph and replay it.
  * The captured calls keep the pointers given here; replaying reads and
  * writes the same buffers. ts_graph_capture_stack captures
@@ -246,6 +291,10 @@ ts_status ts_graph_capture_stack(ts_graph** out, ts_ffn* const* layers, int n_la
                                  int batch, const int32_t* const* active_idx, const int* n_active);
 ts_status ts_graph_capture_moe_stack(ts_graph** out, ts_moe* const* layers, int n_layers,
                                      float* h, int batch);
+/* Captures ts_stack_forward_predicted(layers, preds, n_layers, h, batch, K, lists, .). */
+ts_status ts_graph_capture_stack_predicted(ts_graph** out, ts_ffn* const* layers, ts_predictor* const* preds,
+                                           int n_layers, float* h, int batch, const int* K,
+                                           int32_t* const* lists);
 ts_status ts_graph_launch(ts_graph* g, cudaStream_t stream);
 void ts_graph_destroy(ts_graph* g);
 

@@ -53,6 +53,11 @@ SIGNATURES = {
     "ts_moe_get_error": (I, [P, P]),
     "ts_graph_capture_stack": (I, [PP, P, I, P, I, P, P]),
     "ts_graph_capture_moe_stack": (I, [PP, P, I, P, I]),
+    "ts_predictor_create": (I, [PP, I, I, I, I, P, P, I]),
+    "ts_predictor_destroy": (None, [P]),
+    "ts_predict": (I, [P, P, I, I, P, P, P]),
+    "ts_stack_forward_predicted": (I, [P, P, I, P, I, P, P, P]),
+    "ts_graph_capture_stack_predicted": (I, [PP, P, P, I, P, I, P, P]),
     "ts_graph_launch": (I, [P, P]),
     "ts_graph_destroy": (None, [P]),
 }
@@ -301,6 +306,93 @@ def stack_forward(layers, h: torch.Tensor, active_idx=None, stream=None) -> torc
     return h
 
 
+class Predictor:
+    """Activation predictor of one FFN layer over borrowed ``w1 [r][d]`` and
+    ``w2 [m][r]`` (bf16 or fp32): ``ts_predict`` gives the K neurons with the
+    largest max-over-tokens score of ``w2 relu(w1 x)``, ascending."""
+
+    def __init__(self, w1: torch.Tensor, w2: torch.Tensor, max_batch: int = 1):
+        _dev(w1, "w1")
+        _dev(w2, "w2")
+        if w1.dtype != w2.dtype:
+            raise TypeError("w1 and w2 must share one dtype")
+        self.r, self.d = int(w1.shape[0]), int(w1.shape[1])
+        self.m = int(w2.shape[0])
+        if w2.dim() != 2 or w2.shape[1] != self.r:
+            raise ValueError("w2 must be [m][r] with r = w1.shape[0]")
+        self.dtype, self.max_batch = w1.dtype, int(max_batch)
+        self._keep = (w1, w2)
+        h = ctypes.c_void_p()
+        _check(lib().ts_predictor_create(ctypes.byref(h), self.d, self.r, self.m, _dtype_code(w1),
+                                         w1.data_ptr(), w2.data_ptr(), self.max_batch), "ts_predictor_create")
+        self._h = h
+
+    @property
+    def handle(self) -> ctypes.c_void_p:
+        if self._h is None:
+            raise RuntimeError("handle is closed")
+        return self._h
+
+    def predict(self, x, K: int, out=None, scores=None, stream=None) -> torch.Tensor:
+        """The predicted list (int32 [K], ascending); ``scores`` (fp32
+        [batch][m]), when given, receives every neuron's score."""
+        _dev(x, "x")
+        if x.dtype != self.dtype or x.dim() != 2 or x.shape[1] != self.d:
+            raise ValueError(f"x must be [batch][{self.d}] {self.dtype}")
+        if out is None:
+            out = torch.empty(max(int(K), 1), dtype=torch.int32, device=x.device)
+        _dev(out, "out")
+        if out.dtype != torch.int32 or out.numel() < K:
+            raise ValueError("out must be int32 with at least K entries")
+        sp = None
+        if scores is not None:
+            _dev(scores, "scores")
+            if scores.dtype != torch.float32 or tuple(scores.shape) != (x.shape[0], self.m):
+                raise ValueError(f"scores must be [batch][{self.m}] float32")
+            sp = scores.data_ptr()
+        _check(lib().ts_predict(self.handle, x.data_ptr(), x.shape[0], int(K), out.data_ptr(), sp,
+                                _stream(stream)), "ts_predict")
+        return out[: int(K)]
+
+    def close(self) -> None:
+        if getattr(self, "_h", None) is not None:
+            lib().ts_predictor_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def _predicted_args(layers, preds, K, lists):
+    n = len(layers)
+    if len(preds) != n or len(K) != n or len(lists) != n:
+        raise ValueError("one predictor, K and list buffer per layer")
+    ks = (ctypes.c_int * n)(*[int(k) for k in K])
+    ptrs = (ctypes.c_void_p * n)()
+    for i, (buf, k) in enumerate(zip(lists, K)):
+        _dev(buf, "lists[i]")
+        if buf.dtype != torch.int32 or buf.numel() < max(int(k), 1):
+            raise ValueError("each list buffer must be int32 with at least max(K, 1) entries")
+        ptrs[i] = buf.data_ptr()
+    return _handles(layers), _handles(preds), ks, ptrs
+
+
+def stack_forward_predicted(layers, preds, h: torch.Tensor, K, lists, stream=None) -> torch.Tensor:
+    """``ts_stack_forward_predicted``: each layer predicts its list from
+    rmsnorm(h) into ``lists[l]`` and runs the FFN over it; ``h`` in place."""
+    _dev(h, "h")
+    if h.dtype != torch.float32:
+        raise TypeError("h must be float32")
+    la, pa, ks, ptrs = _predicted_args(layers, preds, K, lists)
+    _check(lib().ts_stack_forward_predicted(_addr(la), _addr(pa), len(layers), h.data_ptr(), h.shape[0],
+                                            _addr(ks), _addr(ptrs), _stream(stream)),
+           "ts_stack_forward_predicted")
+    return h
+
+
 class Moe:
     """Top-k MoE layer over ``Ffn`` experts and a borrowed router ``w_router [E][d]``."""
 
@@ -392,6 +484,16 @@ class Graph:
         _check(lib().ts_graph_capture_stack(ctypes.byref(g), _addr(arr), len(layers), h.data_ptr(),
                                             h.shape[0], _addr(ptrs), _addr(ns)), "ts_graph_capture_stack")
         return cls(g, (list(layers), h, keep))
+
+    @classmethod
+    def stack_predicted(cls, layers, preds, h: torch.Tensor, K, lists) -> "Graph":
+        _dev(h, "h")
+        la, pa, ks, ptrs = _predicted_args(layers, preds, K, lists)
+        g = ctypes.c_void_p()
+        _check(lib().ts_graph_capture_stack_predicted(ctypes.byref(g), _addr(la), _addr(pa), len(layers),
+                                                      h.data_ptr(), h.shape[0], _addr(ks), _addr(ptrs)),
+               "ts_graph_capture_stack_predicted")
+        return cls(g, (list(layers), list(preds), h, ks, ptrs, list(lists)))
 
     @classmethod
     def moe_stack(cls, layers, h: torch.Tensor) -> "Graph":

@@ -20,7 +20,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libtsffn.so")
 SOURCES = ["ts_api.cu", "ts_gate_up.cu", "ts_down.cu", "ts_router.cu", "ts_noalloc.cu", "ts_wide.cu",
-           "ts_topk.cu"]
+           "ts_topk.cu", "ts_predict.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-I", INCLUDE, "-I", CSRC]

@@ -10,6 +10,7 @@
 
 #include "ts_ffn.h"
 #include "ts_kernels.cuh"
+#include "ts_predict.h"
 #include "ts_wide.h"
 
 using namespace tsffn;
@@ -46,7 +47,8 @@ ts_status device_info(DeviceInfo* di) {
         cudaSuccess)
         return TS_ERR_CUDA;
     if (prepare_gate_up(di->optin_smem) != cudaSuccess || prepare_down() != cudaSuccess ||
-        prepare_router() != cudaSuccess || prepare_wide() != cudaSuccess)
+        prepare_router() != cudaSuccess || prepare_wide() != cudaSuccess ||
+        prepare_predict(di->optin_smem) != cudaSuccess)
         return TS_ERR_CUDA;
     return TS_OK;
 }
@@ -132,6 +134,17 @@ struct ts_moe {
     void* xbuf = nullptr;
     int grid[9] = {0};
     int last_batch = 0;
+};
+
+struct ts_predictor {
+    int d = 0, r = 0, m = 0, max_batch = 0;
+    ts_dtype dt = TS_BF16;
+    const void* w1 = nullptr;  // [r][d]
+    const void* w2 = nullptr;  // [m][r]
+    DeviceInfo dev;
+    Arena arena;
+    float* hid = nullptr;      // [kPredMaxSplits][max_batch][r]
+    unsigned* key = nullptr;   // [m]
 };
 
 struct ts_graph {
@@ -386,6 +399,40 @@ ts_status read_status(unsigned* status_dev, cudaStream_t stream) {
     return (v & kStatusBadIndex) ? TS_ERR_BAD_INDEX : TS_OK;
 }
 
+// One layer of the residual stack: h += FFN(rmsnorm(h)) over the layer's
+// rows (all, or the list). `next` is the following layer when it runs dense
+// (its first W_gate rows are then prefetched into L2), else nullptr.
+ts_status stack_layer(ts_ffn* h, const ts_ffn* next, float* hres, int batch, const int32_t* rows, int nr,
+                      cudaStream_t stream) {
+    if (use_wide(h, batch)) {
+        WideLaunch L = wide_launch(h, batch, rows, nr);
+        L.x = h->w_x;
+        L.h = hres;
+        L.residual_out = 1;
+        ts_status st = cuda_status(launch_wide_norm(L, hres, h->w_x, stream, true));
+        if (st == TS_OK) st = cuda_status(launch_wide(L, stream, true));
+        if (st != TS_OK) return st;
+        remember(h, batch, rows, nr);
+        return TS_OK;
+    }
+    FfnLaunch a = ffn_launch(h, batch, rows, nr);
+    a.h = hres;
+    a.norm_from_h = 1;
+    a.residual_out = 1;
+    if (next != nullptr && batch <= kMaxPass && h->dt != TS_INT4) {
+        a.next_wg = next->wg;
+        a.next_n_rows = next->m;
+        a.next_grid = next->grid[pow2_tokens(std::min(kMaxPass, batch))];
+        a.prefetch_rows = kPrefetchRows;
+    }
+    for (int t0 = 0; t0 < batch; t0 += h->pass_max) {
+        ts_status st = run_pass(h, a, t0, std::min(h->pass_max, batch - t0), stream, true, true);
+        if (st != TS_OK) return st;
+    }
+    remember(h, batch, rows, nr);
+    return TS_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -480,36 +527,11 @@ ts_status ts_stack_forward(ts_ffn* const* layers, int n_layers, float* hres, int
         if (st != TS_OK) return st;
     }
     for (int l = 0; l < n_layers; ++l) {
-        ts_ffn* h = layers[l];
         const int32_t* rows = active_idx ? active_idx[l] : nullptr;
-        const int nr = rows ? n_active[l] : 0;
-        if (use_wide(h, batch)) {
-            WideLaunch L = wide_launch(h, batch, rows, nr);
-            L.x = h->w_x;
-            L.h = hres;
-            L.residual_out = 1;
-            ts_status st = cuda_status(launch_wide_norm(L, hres, h->w_x, stream, true));
-            if (st == TS_OK) st = cuda_status(launch_wide(L, stream, true));
-            if (st != TS_OK) return st;
-            remember(h, batch, rows, nr);
-            continue;
-        }
-        FfnLaunch a = ffn_launch(h, batch, rows, nr);
-        a.h = hres;
-        a.norm_from_h = 1;
-        a.residual_out = 1;
         const bool next_dense = l + 1 < n_layers && !(active_idx && active_idx[l + 1]);
-        if (next_dense && batch <= kMaxPass && h->dt != TS_INT4) {
-            a.next_wg = layers[l + 1]->wg;
-            a.next_n_rows = layers[l + 1]->m;
-            a.next_grid = layers[l + 1]->grid[pow2_tokens(std::min(kMaxPass, batch))];
-            a.prefetch_rows = kPrefetchRows;
-        }
-        for (int t0 = 0; t0 < batch; t0 += h->pass_max) {
-            ts_status st = run_pass(h, a, t0, std::min(h->pass_max, batch - t0), stream, true, true);
-            if (st != TS_OK) return st;
-        }
-        remember(h, batch, rows, nr);
+        ts_status st = stack_layer(layers[l], next_dense ? layers[l + 1] : nullptr, hres, batch, rows,
+                                   rows ? n_active[l] : 0, stream);
+        if (st != TS_OK) return st;
     }
     return TS_OK;
 }
@@ -757,6 +779,118 @@ ts_status ts_moe_get_error(ts_moe* h, cudaStream_t stream) {
 // ---------------------------------------------------------------------------
 }  // extern "C"
 
+extern "C" {
+
+ts_status ts_predictor_create(ts_predictor** out, int d, int r, int m, ts_dtype dtype, const void* w1,
+                              const void* w2, int max_batch) {
+    if (out == nullptr) return TS_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (d < 1 || r < 1 || m < 1 || max_batch < 1) return TS_ERR_INVALID_ARG;
+    if (dtype != TS_F32 && dtype != TS_BF16) return TS_ERR_INVALID_ARG;
+    if (!w1 || !w2 || !aligned16(w1) || !aligned16(w2)) return TS_ERR_INVALID_ARG;
+    if (max_batch > kPredMaxBatch || m > (1 << 28)) return TS_ERR_UNSUPPORTED;
+    DeviceInfo dev;
+    ts_status st = device_info(&dev);
+    if (st != TS_OK) return st;
+    if (!predict_supported(elem_size(dtype), d, r, max_batch, dev.optin_smem)) return TS_ERR_UNSUPPORTED;
+    ts_predictor* p = new (std::nothrow) ts_predictor();
+    if (!p) return TS_ERR_OOM;
+    p->d = d;
+    p->r = r;
+    p->m = m;
+    p->max_batch = max_batch;
+    p->dt = dtype;
+    p->w1 = w1;
+    p->w2 = w2;
+    p->dev = dev;
+    const size_t o_h = p->arena.take((size_t)kPredMaxSplits * max_batch * r * sizeof(float));
+    const size_t o_k = p->arena.take((size_t)m * sizeof(unsigned));
+    st = alloc_arena(&p->arena);
+    if (st != TS_OK) {
+        delete p;
+        return st;
+    }
+    p->hid = p->arena.at<float>(o_h);
+    p->key = p->arena.at<unsigned>(o_k);
+    *out = p;
+    return TS_OK;
+}
+
+void ts_predictor_destroy(ts_predictor* p) {
+    if (!p) return;
+    if (p->arena.base) cudaFree(p->arena.base);
+    delete p;
+}
+
+}  // extern "C"
+
+namespace {
+
+PredictLaunch predict_launch(const ts_predictor* p, int batch, int K, int32_t* list, float* scores) {
+    PredictLaunch q;
+    memset(&q, 0, sizeof q);
+    q.d = p->d;
+    q.r = p->r;
+    q.m = p->m;
+    q.batch = batch;
+    q.w1 = p->w1;
+    q.w2 = p->w2;
+    q.hid = p->hid;
+    q.key = p->key;
+    q.scores = scores;
+    q.K = K;
+    q.list = list;
+    predict_geometry(&q, elem_size(p->dt), p->dev.num_sms);
+    return q;
+}
+
+}  // namespace
+
+extern "C" {
+
+ts_status ts_predict(ts_predictor* p, const void* x, int batch, int K, int32_t* list, float* scores,
+                     cudaStream_t stream) {
+    if (!p || batch < 0 || batch > p->max_batch || K < 0 || K > p->m) return TS_ERR_INVALID_ARG;
+    if (batch == 0 || K == 0) return TS_OK;
+    if (!x || !list || ((uintptr_t)x & (act_size(p->dt) - 1)) != 0 || ((uintptr_t)list & 3u) != 0)
+        return TS_ERR_INVALID_ARG;
+    PredictLaunch q = predict_launch(p, batch, K, list, scores);
+    q.x = x;
+    return cuda_status(launch_predict(q, elem_size(p->dt), stream, true));
+}
+
+ts_status ts_stack_forward_predicted(ts_ffn* const* layers, ts_predictor* const* preds, int n_layers,
+                                     float* hres, int batch, const int* K, int32_t* const* lists,
+                                     cudaStream_t stream) {
+    if (!layers || !preds || n_layers < 0 || !hres || batch < 0) return TS_ERR_INVALID_ARG;
+    if (batch == 0 || n_layers == 0) return TS_OK;
+    if (!K || !lists) return TS_ERR_INVALID_ARG;
+    for (int l = 0; l < n_layers; ++l) {
+        const ts_ffn* h = layers[l];
+        const ts_predictor* p = preds[l];
+        if (!h || !p || h->d != layers[0]->d || h->dt != layers[0]->dt || batch > h->max_batch)
+            return TS_ERR_INVALID_ARG;
+        if (p->d != h->d || p->m != h->m || p->dt != act_dtype(h->dt) || batch > p->max_batch)
+            return TS_ERR_INVALID_ARG;
+        if (K[l] < 0 || K[l] > h->m || !lists[l] || ((uintptr_t)lists[l] & 3u) != 0) return TS_ERR_INVALID_ARG;
+    }
+    for (int l = 0; l < n_layers; ++l) {
+        ts_ffn* h = layers[l];
+        if (K[l] == 0) {  // an empty list: the layer adds nothing
+            remember(h, batch, lists[l], 0);
+            continue;
+        }
+        PredictLaunch q = predict_launch(preds[l], batch, K[l], lists[l], nullptr);
+        q.h = hres;
+        ts_status st = cuda_status(launch_predict(q, elem_size(preds[l]->dt), stream, true));
+        if (st == TS_OK) st = stack_layer(h, nullptr, hres, batch, lists[l], K[l], stream);
+        if (st != TS_OK) return st;
+    }
+    return TS_OK;
+}
+
+}  // extern "C"
+
 namespace {
 
 template <typename F>
@@ -806,6 +940,14 @@ ts_status ts_graph_capture_stack(ts_graph** out, ts_ffn* const* layers, int n_la
 ts_status ts_graph_capture_moe_stack(ts_graph** out, ts_moe* const* layers, int n_layers, float* h,
                                      int batch) {
     return capture(out, [&](cudaStream_t s) { return ts_moe_stack_forward(layers, n_layers, h, batch, s); });
+}
+
+ts_status ts_graph_capture_stack_predicted(ts_graph** out, ts_ffn* const* layers, ts_predictor* const* preds,
+                                           int n_layers, float* h, int batch, const int* K,
+                                           int32_t* const* lists) {
+    return capture(out, [&](cudaStream_t s) {
+        return ts_stack_forward_predicted(layers, preds, n_layers, h, batch, K, lists, s);
+    });
 }
 
 ts_status ts_graph_launch(ts_graph* g, cudaStream_t stream) {

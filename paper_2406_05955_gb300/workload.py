@@ -240,6 +240,11 @@ WORKLOADS = {
         d=MISTRAL_D, m=MISTRAL_M, dtype="bf16", batch=1, layers=N_LAYERS, activation=0.10,
         list_len=1434, zipf_s=1.1, seed=1000,
         desc="predictor-driven mode: per-layer sorted lists of 1434 neurons (Zipf 1.1 over hotness)"),
+    "mistral7b-ffn-stack-bf16-b1-prednet": dict(
+        d=MISTRAL_D, m=MISTRAL_M, dtype="bf16", batch=1, layers=N_LAYERS, activation=0.10, rank=512, k=1434,
+        seed=1000,
+        desc="per-layer predictor network (two-layer ReLU MLP, rank 512) choosing 1434 neurons (10%) "
+             "for the FFN's predictor mode, 32 layers, batch 1"),
 }
 
 
