@@ -750,23 +750,9 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up(const F
     const int x_tok0 = a.route ? 0 : a.tok0;
     for (int t = 0; t < n_x; ++t) {
         float* xrow = xs + (size_t)t * cfg.xs_stride;
-        if (a.norm_from_h) {
-            const float* hr = a.h + (size_t)(x_tok0 + t) * a.d;
-            float ss = 0.0f;
-            for (int i = ctid; i < a.d; i += cthreads) ss = fmaf(hr[i], hr[i], ss);
-            ss = warp_sum(ss);
-            if (lane == 0) sh.red[warp - 1] = ss;
-            named_bar_sync(1, cthreads);
-            float tot = 0.0f;
-            for (int w = 0; w < GateUpWarps<NT>::C; ++w) tot += sh.red[w];
-            const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)a.d), 1e-5f));
-            for (int i = ctid; i < a.d; i += cthreads)
-                xrow[xs_index<T>(i)] = (i == a.d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hr[i], rms));
-            named_bar_sync(1, cthreads);
-        } else {
-            for (int i = ctid; i < a.d; i += cthreads)
-                xrow[xs_index<T>(i)] = Vec<T>::load1(a.x, (size_t)(x_tok0 + t) * a.d + i);
-        }
+        stage_act_row<T>(a.norm_from_h ? a.h + (size_t)(x_tok0 + t) * a.d : nullptr,
+                         static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d, a.d, ctid, cthreads, sh.red,
+                         [&](int i, float v) { xrow[xs_index<T>(i)] = v; });
     }
     named_bar_sync(1, cthreads);
     consume<T, NT>(a, sh, ring, xs, cfg, warp - 1, lane);
@@ -1072,22 +1058,10 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_mma(con
         __nv_bfloat16* xrow = reinterpret_cast<__nv_bfloat16*>(xb + (size_t)t * mc.x_stride);
         if (t >= n_x) {
             for (int i = ctid; i < a.d; i += cthreads) xrow[i] = __float2bfloat16_rn(0.0f);
-        } else if (a.norm_from_h) {
-            const float* hr = a.h + (size_t)(x_tok0 + t) * a.d;
-            float ss = 0.0f;
-            for (int i = ctid; i < a.d; i += cthreads) ss = fmaf(hr[i], hr[i], ss);
-            ss = warp_sum(ss);
-            if (lane == 0) sh.red[warp - 1] = ss;
-            named_bar_sync(1, cthreads);
-            float tot = 0.0f;
-            for (int w = 0; w < C; ++w) tot += sh.red[w];
-            const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)a.d), 1e-5f));
-            for (int i = ctid; i < a.d; i += cthreads)
-                xrow[i] = __float2bfloat16_rn((i == a.d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hr[i], rms)));
-            named_bar_sync(1, cthreads);
         } else {
-            const T* xr = static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d;
-            for (int i = ctid; i < a.d; i += cthreads) xrow[i] = xr[i];
+            stage_act_row<T>(a.norm_from_h ? a.h + (size_t)(x_tok0 + t) * a.d : nullptr,
+                             static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d, a.d, ctid, cthreads, sh.red,
+                             [&](int i, float v) { xrow[i] = __float2bfloat16_rn(v); });
         }
     }
     named_bar_sync(1, cthreads);
@@ -1334,17 +1308,19 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
             return true;
         }
     };
-    // The weights do not depend on the activations: the first round's
-    // chunks and each warp's first gate rows are set going before the
-    // activations are staged (and, for the dense layer, before the wait for
-    // the kernel that writes them).
+    // The weights do not depend on the activations: each warp's first gate
+    // rows are set going while the activations are staged, just after the
+    // activation loads are issued (so those loads do not queue behind the
+    // row copies).
     int c_first = 0;
     unsigned r_first = 0u;
     setup(0, min(kQ4Round, n_local));
     named_bar_sync(1, cthreads);
-    const bool have_first = claim(0, 2 * min(kQ4Round, n_local), c_first, r_first);
-    if (have_first) issue(kTaskGate, c_first, r_first, 0);
-    stage();
+    bool have_first = false;
+    stage([&]() {
+        have_first = claim(0, 2 * min(kQ4Round, n_local), c_first, r_first);
+        if (have_first) issue(kTaskGate, c_first, r_first, 0);
+    });
 
     for (int base = 0; base < n_local; base += kQ4Round) {
         const int nr = min(kQ4Round, n_local - base);
@@ -1463,32 +1439,29 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
     const int x_tok0 = a.route ? 0 : a.tok0;
     const int dq = a.d / 4;
     auto xpos = [&](int i) { return (i / dq) * (dq + kQ4QuarterPad / 2) + i % dq; };  // bf16 index in a row
-    auto stage = [&]() {
-    if (early) pdl_wait();
-    for (int t = 0; t < NT; ++t) {
-        __nv_bfloat16* xrow = reinterpret_cast<__nv_bfloat16*>(xb + (size_t)t * mc.x_stride);
-        if (t >= n_x) {
-            for (int i = ctid; i < a.d; i += cthreads) xrow[xpos(i)] = __float2bfloat16_rn(0.0f);
-        } else if (a.norm_from_h) {
-            const float* hr = a.h + (size_t)(x_tok0 + t) * a.d;
-            float ss = 0.0f;
-            for (int i = ctid; i < a.d; i += cthreads) ss = fmaf(hr[i], hr[i], ss);
-            ss = warp_sum(ss);
-            if (lane == 0) sh.red[warp - 1] = ss;
-            named_bar_sync(1, cthreads);
-            float tot = 0.0f;
-            for (int w = 0; w < C; ++w) tot += sh.red[w];
-            const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)a.d), 1e-5f));
-            for (int i = ctid; i < a.d; i += cthreads)
-                xrow[xpos(i)] =
-                    __float2bfloat16_rn((i == a.d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hr[i], rms)));
-            named_bar_sync(1, cthreads);
-        } else {
-            const T* xr = static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d;
-            for (int i = ctid; i < a.d; i += cthreads) xrow[xpos(i)] = xr[i];
+    // Stage the activations; first_rows() (the first weight-row copies) runs
+    // once, right after the first activation loads are issued.
+    auto stage = [&](auto&& first_rows) {
+        if (early) pdl_wait();
+        bool started = false;
+        auto once = [&]() {
+            if (!started) {
+                started = true;
+                first_rows();
+            }
+        };
+        for (int t = 0; t < NT; ++t) {
+            __nv_bfloat16* xrow = reinterpret_cast<__nv_bfloat16*>(xb + (size_t)t * mc.x_stride);
+            if (t >= n_x) {
+                for (int i = ctid; i < a.d; i += cthreads) xrow[xpos(i)] = __float2bfloat16_rn(0.0f);
+            } else {
+                stage_act_row<T>(a.norm_from_h ? a.h + (size_t)(x_tok0 + t) * a.d : nullptr,
+                                 static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d, a.d, ctid, cthreads,
+                                 sh.red, [&](int i, float v) { xrow[xpos(i)] = __float2bfloat16_rn(v); }, once);
+            }
         }
-    }
-    named_bar_sync(1, cthreads);
+        once();
+        named_bar_sync(1, cthreads);
     };
     consume_q4w<NT>(a, sh, ring, xb, tab, mc, i0, i1, n_chunks, warp - 1, lane, stage);
     down_partial<T, NT, true>(a, sh, i0, i1, n_chunks, warp - 1, lane);
@@ -1636,18 +1609,20 @@ __device__ void consume_rows(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned 
     };
 
     // The weights do not depend on the activations: the first round's rows
-    // are set going before the activations are staged (and, for the dense
-    // layer, before the wait for the kernel that writes them).
+    // are set going while the activations are staged, just after the
+    // activation loads are issued (so those loads do not queue behind the
+    // row copies).
     int qc[kRowsMaxAhead + 1], qr[kRowsMaxAhead + 1];  // claimed rows, oldest first
     int n_q = 0, head_slot = 0;
     const int nr0 = min(kQ4Round, n_local);
     setup(0, nr0);
     named_bar_sync(1, cthreads);
-    while (n_q < P && claim(0, kChunk * nr0, qc[n_q], qr[n_q])) {
-        issue(kTaskGate, qc[n_q], qr[n_q], n_q);
-        ++n_q;
-    }
-    stage();
+    stage([&]() {
+        while (n_q < P && claim(0, kChunk * nr0, qc[n_q], qr[n_q])) {
+            issue(kTaskGate, qc[n_q], qr[n_q], n_q);
+            ++n_q;
+        }
+    });
 
     for (int base = 0; base < n_local; base += kQ4Round) {
         const int nr = min(kQ4Round, n_local - base);
@@ -1752,28 +1727,24 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(co
     const int ctid = threadIdx.x - kWarp;
     const int cthreads = C * kWarp;
     const int x_tok0 = a.route ? 0 : a.tok0;
-    auto stage = [&]() {
+    // Stage the activations; first_rows() (the first weight-row copies) runs
+    // once, right after the first activation loads are issued.
+    auto stage = [&](auto&& first_rows) {
         if (early) pdl_wait();
+        bool started = false;
+        auto once = [&]() {
+            if (!started) {
+                started = true;
+                first_rows();
+            }
+        };
         for (int t = 0; t < n_x; ++t) {
             float* xrow = xs + (size_t)t * rc.xs_stride;
-            if (a.norm_from_h) {
-                const float* hr = a.h + (size_t)(x_tok0 + t) * a.d;
-                float ss = 0.0f;
-                for (int i = ctid; i < a.d; i += cthreads) ss = fmaf(hr[i], hr[i], ss);
-                ss = warp_sum(ss);
-                if (lane == 0) sh.red[warp - 1] = ss;
-                named_bar_sync(1, cthreads);
-                float tot = 0.0f;
-                for (int w = 0; w < C; ++w) tot += sh.red[w];
-                const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)a.d), 1e-5f));
-                for (int i = ctid; i < a.d; i += cthreads)
-                    xrow[xs_index<T>(i)] = (i == a.d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hr[i], rms));
-                named_bar_sync(1, cthreads);
-            } else {
-                for (int i = ctid; i < a.d; i += cthreads)
-                    xrow[xs_index<T>(i)] = Vec<T>::load1(a.x, (size_t)(x_tok0 + t) * a.d + i);
-            }
+            stage_act_row<T>(a.norm_from_h ? a.h + (size_t)(x_tok0 + t) * a.d : nullptr,
+                             static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d, a.d, ctid, cthreads, sh.red,
+                             [&](int i, float v) { xrow[xs_index<T>(i)] = v; }, once);
         }
+        once();
         named_bar_sync(1, cthreads);
     };
     consume_rows<T, NT>(a, sh, ring, xs, tab, ulist, rc, i0, i1, n_chunks, warp - 1, lane, stage);

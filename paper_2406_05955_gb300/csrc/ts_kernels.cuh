@@ -188,6 +188,12 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity) {
         if (global_ns() - t0 > kWaitLimitNs) return false;
     return true;
 }
+// Order this thread's earlier generic-proxy accesses to shared memory before
+// its later async-proxy (bulk copy) accesses, e.g. reads of a slot before a
+// copy that overwrites it.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
 // 1-D bulk copy global -> this CTA's shared memory, completing on `bar`.
 __device__ __forceinline__ void tma_load_1d(void* dst, const void* src, unsigned bytes, uint64_t* bar) {
     asm volatile(
@@ -304,6 +310,105 @@ __device__ __forceinline__ void resolve_experts(const FfnLaunch& a, ExpertSets& 
         }
     }
     __syncthreads();
+}
+
+// One activation row of a gate+up CTA's consumer threads (ctid < cthreads,
+// cwarp = ctid / 32, named barrier 1), handed element by element to
+// put(i, v): x = round(h / sqrt(mean(h^2) + 1e-5)) with x[d-1] = 1 when
+// `h` is given (stack mode), else the row of x as stored. Every global load
+// of a group of kStageVec 16-byte vectors per thread is issued before any is
+// used, so the row arrives in one memory round trip instead of one per
+// element; for d <= 4 * kStageVec * cthreads the h values stay in registers
+// between the sum of squares and the division. The sum of squares runs in a
+// fixed order (per thread, then the warp tree, then warps in order), so every
+// CTA computes the same bits. `red` holds one float per consumer warp.
+// `after_loads()` runs once, right after the first group's loads are
+// issued and before any of them is used: work placed there (such as the
+// first weight-row copies) queues behind the activations instead of ahead.
+constexpr int kStageVec = 4;
+
+struct NoAfterLoads {
+    __device__ __forceinline__ void operator()() const {}
+};
+
+template <typename T, typename Put, typename After = NoAfterLoads>
+__device__ __forceinline__ void stage_act_row(const float* __restrict__ h, const void* x, int d, int ctid,
+                                              int cthreads, float* red, Put put, After after_loads = After()) {
+    const int lane = ctid & 31, cwarp = ctid >> 5, nw = cthreads >> 5;
+    if (h != nullptr) {
+        const bool vec = (d % 4) == 0 && (reinterpret_cast<uintptr_t>(h) & 15u) == 0;
+        const int d4 = vec ? d / 4 : 0;
+        const int group = kStageVec * cthreads;  // float4 per group
+        float4 v[kStageVec];
+        float ss = 0.0f;
+        if (d4 == 0) after_loads();
+        for (int g0 = 0; g0 < d4; g0 += group) {
+#pragma unroll
+            for (int k = 0; k < kStageVec; ++k) {
+                const int q = g0 + ctid + k * cthreads;
+                v[k] = q < d4 ? *reinterpret_cast<const float4*>(h + 4 * (size_t)q) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            if (g0 == 0) after_loads();
+#pragma unroll
+            for (int k = 0; k < kStageVec; ++k) {
+                ss = fmaf(v[k].x, v[k].x, ss);
+                ss = fmaf(v[k].y, v[k].y, ss);
+                ss = fmaf(v[k].z, v[k].z, ss);
+                ss = fmaf(v[k].w, v[k].w, ss);
+            }
+        }
+        for (int i = 4 * d4 + ctid; i < d; i += cthreads) ss = fmaf(h[i], h[i], ss);  // rows with d % 4 != 0
+        ss = warp_sum(ss);
+        if (lane == 0) red[cwarp] = ss;
+        named_bar_sync(1, cthreads);
+        float tot = 0.0f;
+        for (int w = 0; w < nw; ++w) tot += red[w];
+        const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)d), 1e-5f));
+        auto norm = [&](int i, float hv) { return (i == d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hv, rms)); };
+        const bool kept = d4 <= group;  // the single group is still in registers
+        for (int g0 = 0; g0 < d4; g0 += group) {
+#pragma unroll
+            for (int k = 0; k < kStageVec; ++k) {
+                const int q = g0 + ctid + k * cthreads;
+                if (q < d4) {
+                    const float4 w = kept ? v[k] : *reinterpret_cast<const float4*>(h + 4 * (size_t)q);
+                    put(4 * q, norm(4 * q, w.x));
+                    put(4 * q + 1, norm(4 * q + 1, w.y));
+                    put(4 * q + 2, norm(4 * q + 2, w.z));
+                    put(4 * q + 3, norm(4 * q + 3, w.w));
+                }
+            }
+        }
+        for (int i = 4 * d4 + ctid; i < d; i += cthreads) put(i, norm(i, h[i]));
+        named_bar_sync(1, cthreads);  // red[] is reused by the next row
+    } else {
+        constexpr int N = Vec<T>::N;  // elements per 16-byte vector
+        const bool vec = (d % N) == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+        const int dv = vec ? d / N : 0;
+        const int group = kStageVec * cthreads;
+        if (dv == 0) after_loads();
+        for (int g0 = 0; g0 < dv; g0 += group) {
+            uint4 w[kStageVec];
+#pragma unroll
+            for (int k = 0; k < kStageVec; ++k) {
+                const int q = g0 + ctid + k * cthreads;
+                w[k] = q < dv ? *reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(x) + 16 * (size_t)q)
+                              : make_uint4(0u, 0u, 0u, 0u);
+            }
+            if (g0 == 0) after_loads();
+#pragma unroll
+            for (int k = 0; k < kStageVec; ++k) {
+                const int q = g0 + ctid + k * cthreads;
+                if (q < dv) {
+                    float f[N];
+                    Vec<T>::unpack(w[k], f);
+#pragma unroll
+                    for (int e = 0; e < N; ++e) put(N * q + e, f[e]);
+                }
+            }
+        }
+        for (int i = N * dv + ctid; i < d; i += cthreads) put(i, Vec<T>::load1(x, (size_t)i));
+    }
 }
 
 // x = round(h / sqrt(mean(h^2) + 1e-5)), x[d-1] = 1, into shared memory.
