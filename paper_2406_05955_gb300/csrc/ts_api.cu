@@ -145,6 +145,7 @@ struct ts_predictor {
     Arena arena;
     float* hid = nullptr;      // [kPredMaxSplits][max_batch][r]
     unsigned* key = nullptr;   // [m]
+    unsigned* hist = nullptr;  // [kPredHistParts][kPredHistBins]
 };
 
 struct ts_graph {
@@ -805,6 +806,7 @@ ts_status ts_predictor_create(ts_predictor** out, int d, int r, int m, ts_dtype 
     p->dev = dev;
     const size_t o_h = p->arena.take((size_t)kPredMaxSplits * max_batch * r * sizeof(float));
     const size_t o_k = p->arena.take((size_t)m * sizeof(unsigned));
+    const size_t o_b = p->arena.take((size_t)kPredHistParts * kPredHistBins * sizeof(unsigned));
     st = alloc_arena(&p->arena);
     if (st != TS_OK) {
         delete p;
@@ -812,6 +814,7 @@ ts_status ts_predictor_create(ts_predictor** out, int d, int r, int m, ts_dtype 
     }
     p->hid = p->arena.at<float>(o_h);
     p->key = p->arena.at<unsigned>(o_k);
+    p->hist = p->arena.at<unsigned>(o_b);
     *out = p;
     return TS_OK;
 }
@@ -837,6 +840,7 @@ PredictLaunch predict_launch(const ts_predictor* p, int batch, int K, int32_t* l
     q.w2 = p->w2;
     q.hid = p->hid;
     q.key = p->key;
+    q.hist = p->hist;
     q.scores = scores;
     q.K = K;
     q.list = list;

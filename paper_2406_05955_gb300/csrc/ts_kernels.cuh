@@ -411,25 +411,13 @@ __device__ __forceinline__ void stage_act_row(const float* __restrict__ h, const
     }
 }
 
-// x = round(h / sqrt(mean(h^2) + 1e-5)), x[d-1] = 1, into shared memory.
+// x = round(h / sqrt(mean(h^2) + 1e-5)), x[d-1] = 1, into shared memory, by
+// the whole block (blockDim.x a multiple of 32, `red` one float per warp).
 // Every block computes the same bits (fixed per-thread order, fixed tree).
 template <typename T>
 __device__ __forceinline__ void block_rmsnorm(const float* __restrict__ h, int d, float* __restrict__ out,
-                              float* red) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-    float ss = 0.0f;
-    for (int i = threadIdx.x; i < d; i += blockDim.x) {
-        const float v = h[i];
-        ss = fmaf(v, v, ss);
-    }
-    ss = warp_sum(ss);
-    if (lane == 0) red[warp] = ss;
-    __syncthreads();
-    float tot = 0.0f;
-    for (int w = 0; w < nw; ++w) tot += red[w];
-    const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)d), 1e-5f));
-    for (int i = threadIdx.x; i < d; i += blockDim.x)
-        out[i] = (i == d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(h[i], rms));
+                                              float* red) {
+    stage_act_row<T>(h, nullptr, d, (int)threadIdx.x, (int)blockDim.x, red, [&](int i, float v) { out[i] = v; });
     __syncthreads();
 }
 

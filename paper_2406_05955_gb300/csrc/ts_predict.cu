@@ -57,6 +57,10 @@ __global__ void __launch_bounds__(kPredThreads) k_pred_hidden(const PredictLaunc
     __shared__ float red[kPredWarps];
     pdl_wait();
     pdl_launch_dependents();
+    // the select of the previous prediction has finished with the histogram
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < kPredHistParts * kPredHistBins;
+         i += gridDim.x * blockDim.x)
+        p.hist[i] = 0u;
     constexpr int N = Vec<T>::N;
     const int d = p.d;
     if (p.h != nullptr) {
@@ -176,7 +180,11 @@ __global__ void __launch_bounds__(kPredThreads) k_pred_score(const PredictLaunch
                     if (p.scores != nullptr && lane == 0 && j < m) p.scores[(size_t)t * m + j] = sv;
                 }
             }
-            if (lane == 0 && j < m) p.key[j] = order_key(best);
+            if (lane == 0 && j < m) {
+                const unsigned k = order_key(best);
+                p.key[j] = k;
+                atomicAdd(&p.hist[(blockIdx.x % kPredHistParts) * kPredHistBins + (k >> 20)], 1u);
+            }
         }
     }
 }
@@ -294,6 +302,153 @@ __global__ void __launch_bounds__(kSelThreads) k_pred_select(const PredictLaunch
     }
 }
 
+// Exclusive prefix sums over the block's threads (thread order) of two
+// counts at once, and their totals. Whole block; s_a, s_b hold kSelWarps ints.
+__device__ __forceinline__ void block_scan2(int a, int b, int& ea, int& eb, int& ta, int& tb, int* s_a, int* s_b,
+                                            int* s_tot) {
+    const unsigned full = 0xffffffffu;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int ia = a, ib = b;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int na = __shfl_up_sync(full, ia, o), nb = __shfl_up_sync(full, ib, o);
+        if (lane >= o) {
+            ia += na;
+            ib += nb;
+        }
+    }
+    if (lane == 31) {
+        s_a[warp] = ia;
+        s_b[warp] = ib;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        int wa = s_a[lane], wb = s_b[lane];
+        const int wa0 = wa, wb0 = wb;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int na = __shfl_up_sync(full, wa, o), nb = __shfl_up_sync(full, wb, o);
+            if (lane >= o) {
+                wa += na;
+                wb += nb;
+            }
+        }
+        s_a[lane] = wa - wa0;
+        s_b[lane] = wb - wb0;
+        if (lane == 31) {
+            s_tot[0] = wa;
+            s_tot[1] = wb;
+        }
+    }
+    __syncthreads();
+    ea = s_a[warp] + ia - a;
+    eb = s_b[warp] + ib - b;
+    ta = s_tot[0];
+    tb = s_tot[1];
+    __syncthreads();  // s_a, s_b, s_tot may be reused
+}
+
+// The same selection for m <= kSelThreads * kSelKeys, led by the score
+// kernel's histogram of the keys' top 12 bits. Thread t holds ids
+// t*per .. t*per+per-1 in registers, so thread order is id order.
+//   1. Thread t sums the copies of bins 4095-4t .. 4092-4t (highest first); a block scan
+//      of their counts finds the bin B holding the K-th largest key and the
+//      number of keys above it.
+//   2. The keys in bin B (usually a few hundred) are compacted into shared
+//      memory, and the (K - above)-th largest of their low 20 bits is found
+//      bit by bit from the top (keep bit b if enough candidates are >= the
+//      prefix with b set), which gives the K-th largest key T.
+//   3. A block scan of the per-thread counts of keys > T and == T places
+//      every kept id in ascending order.
+// Absent ids hold key 0 and are never counted.
+constexpr int kSelKeys = 16;
+
+__global__ void __launch_bounds__(kSelThreads) k_pred_select_hist(const PredictLaunch p) {
+    extern __shared__ unsigned cand[];  // [m] low 20 bits of the keys in bin B
+    __shared__ int s_a[kSelWarps], s_b[kSelWarps], s_tot[2];
+    __shared__ int s_cnt[2][kSelWarps];
+    __shared__ int s_bin, s_above;
+    pdl_wait();
+    pdl_launch_dependents();
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int m = p.m, K = p.K;
+    const unsigned full = 0xffffffffu;
+    const int per = (m + kSelThreads - 1) / kSelThreads;  // <= kSelKeys
+    const int i0 = tid * per;
+    unsigned key[kSelKeys];
+#pragma unroll
+    for (int q = 0; q < kSelKeys; ++q) key[q] = (q < per && i0 + q < m) ? p.key[i0 + q] : 0u;
+    constexpr int BPT = kPredHistBins / kSelThreads;  // bins per thread
+    int hv[BPT], hsum = 0;
+#pragma unroll
+    for (int q = 0; q < BPT; ++q) {
+        hv[q] = 0;
+#pragma unroll
+        for (int part = 0; part < kPredHistParts; ++part)
+            hv[q] += (int)p.hist[part * kPredHistBins + kPredHistBins - 1 - (BPT * tid + q)];
+        hsum += hv[q];
+    }
+    int above, unused, htot, unused2;
+    block_scan2(hsum, 0, above, unused, htot, unused2, s_a, s_b, s_tot);
+#pragma unroll
+    for (int q = 0; q < BPT; ++q) {
+        if (above < K && K <= above + hv[q]) {  // exactly one bin of one thread
+            s_bin = kPredHistBins - 1 - (BPT * tid + q);
+            s_above = above;
+        }
+        above += hv[q];
+    }
+    __syncthreads();
+    const unsigned B = (unsigned)s_bin;
+    const int need_in_bin = K - s_above;
+
+    int c = 0;
+#pragma unroll
+    for (int q = 0; q < kSelKeys; ++q) c += (key[q] != 0u && (key[q] >> 20) == B) ? 1 : 0;
+    int off, unused3, n_c, unused4;
+    block_scan2(c, 0, off, unused3, n_c, unused4, s_a, s_b, s_tot);
+#pragma unroll
+    for (int q = 0; q < kSelKeys; ++q)
+        if (key[q] != 0u && (key[q] >> 20) == B) cand[off++] = key[q] & 0xfffffu;
+    __syncthreads();
+
+    unsigned L = 0u;
+    for (int b = 19; b >= 0; --b) {
+        const unsigned cv = L | (1u << b);
+        int cnt = 0;
+        for (int i = tid; i < n_c; i += kSelThreads) cnt += cand[i] >= cv ? 1 : 0;
+        cnt = (int)__reduce_add_sync(full, (unsigned)cnt);
+        // two buffers: a step's writes cannot meet the previous step's reads
+        if (lane == 0) s_cnt[b & 1][warp] = cnt;
+        __syncthreads();
+        const int tot = (int)__reduce_add_sync(full, (unsigned)s_cnt[b & 1][lane]);
+        if (tot >= need_in_bin) L = cv;
+    }
+    const unsigned T = (B << 20) | L;
+
+    int gt = 0, eq = 0;
+#pragma unroll
+    for (int q = 0; q < kSelKeys; ++q) {
+        gt += (key[q] != 0u && key[q] > T) ? 1 : 0;
+        eq += (key[q] != 0u && key[q] == T) ? 1 : 0;
+    }
+    int run_gt, run_eq, total_gt, total_eq;
+    block_scan2(gt, eq, run_gt, run_eq, total_gt, total_eq, s_a, s_b, s_tot);
+    const int need = K - total_gt;  // ids with key == T that are kept (the first ones)
+#pragma unroll
+    for (int q = 0; q < kSelKeys; ++q) {
+        const unsigned k = key[q];
+        if (k == 0u) continue;
+        if (k > T) {
+            p.list[run_gt + min(run_eq, need)] = i0 + q;
+            ++run_gt;
+        } else if (k == T) {
+            if (run_eq < need) p.list[run_gt + run_eq] = i0 + q;
+            ++run_eq;
+        }
+    }
+}
+
 template <typename T, int NB>
 cudaError_t launch_nb(const PredictLaunch& p, cudaLaunchConfig_t lc) {
     constexpr int N = Vec<T>::N;
@@ -312,9 +467,13 @@ cudaError_t launch_nb(const PredictLaunch& p, cudaLaunchConfig_t lc) {
         default: return cudaErrorInvalidValue;
     }
     if (e != cudaSuccess) return e;
-    const int staged = (size_t)p.m * sizeof(unsigned) <= (size_t)g_sel_smem;
     lc.gridDim = dim3(1);
     lc.blockDim = dim3(kSelThreads);
+    if (p.m <= kSelThreads * kSelKeys) {
+        lc.dynamicSmemBytes = (size_t)p.m * sizeof(unsigned);
+        return cudaLaunchKernelEx(&lc, k_pred_select_hist, p);
+    }
+    const int staged = (size_t)p.m * sizeof(unsigned) <= (size_t)g_sel_smem;
     lc.dynamicSmemBytes = staged ? (size_t)p.m * sizeof(unsigned) : 0;
     return cudaLaunchKernelEx(&lc, k_pred_select, p, staged);
 }
@@ -389,6 +548,9 @@ cudaError_t prepare_predict(int optin_smem) {
     const int sel_smem = std::min(kSelSmemMax, optin_smem - kSmemSlack);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(k_pred_select, cudaFuncAttributeMaxDynamicSharedMemorySize, sel_smem);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_pred_select_hist, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kSelThreads * kSelKeys * (int)sizeof(unsigned));
     if (e == cudaSuccess) g_sel_smem = sel_smem;
     return e;
 }

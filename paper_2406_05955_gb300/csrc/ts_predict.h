@@ -12,6 +12,8 @@ namespace tsffn {
 
 constexpr int kPredMaxBatch = 8;   // tokens per prediction (x rows held in shared memory)
 constexpr int kPredMaxSplits = 8;  // K-splits of a W1 row
+constexpr int kPredHistBins = 4096;  // histogram of the keys' top 12 bits
+constexpr int kPredHistParts = 8;    // copies of it, by score CTA, to spread the atomics
 
 struct PredictLaunch {
     int d, r, m, batch;
@@ -24,6 +26,9 @@ struct PredictLaunch {
     int hid_grid;        // CTAs of the hidden-layer kernel
     int score_grid;      // CTAs of the score kernel
     unsigned* key;       // [m] order-preserving bits of max_t s[t][j]
+    unsigned* hist;      // [kPredHistParts][kPredHistBins] count of keys per top-12-bit value, one
+                         // copy per score-CTA residue mod kPredHistParts (cleared by the
+                         // hidden-layer kernel, filled by the score kernel, summed by the select)
     float* scores;       // [batch][m] fp32 scores, or nullptr
     int K;               // list length, 1 <= K <= m
     int32_t* list;       // [K] out: ascending neuron ids
