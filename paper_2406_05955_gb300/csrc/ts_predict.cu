@@ -55,14 +55,32 @@ template <typename T, int NB>
 __global__ void __launch_bounds__(kPredThreads) k_pred_hidden(const PredictLaunch p) {
     extern __shared__ __align__(16) float xs[];  // [NB][d]
     __shared__ float red[kPredWarps];
-    pdl_wait();
+    constexpr int N = Vec<T>::N;
+    const int d = p.d;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int steps = d / (kWarp * N) / p.splits;  // 16-byte vectors per lane per piece
+    const int seg = steps * kWarp * N;
+    const int total = p.r * p.splits;
+    auto wrow_of = [&](int piece) {
+        const int sp = piece / p.r, row = piece - sp * p.r;
+        return static_cast<const T*>(p.w1) + (size_t)row * d + (size_t)sp * seg + lane * N;
+    };
+    // W1 does not depend on earlier kernels: the first vectors of this warp's
+    // first piece are loaded before the wait, while the previous kernel ends.
+    int piece = blockIdx.x * kPredWarps + warp;
+    uint4 v[8];
+    if (piece < total) {
+        const T* wrow = wrow_of(piece);
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+            v[u] = u < steps ? ld_stream(wrow + (size_t)u * kWarp * N) : make_uint4(0u, 0u, 0u, 0u);
+    }
     pdl_launch_dependents();
+    pdl_wait();
     // the select of the previous prediction has finished with the histogram
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < kPredHistParts * kPredHistBins;
          i += gridDim.x * blockDim.x)
         p.hist[i] = 0u;
-    constexpr int N = Vec<T>::N;
-    const int d = p.d;
     if (p.h != nullptr) {
         for (int t = 0; t < NB; ++t) {
             if (t < p.batch) {
@@ -77,22 +95,22 @@ __global__ void __launch_bounds__(kPredThreads) k_pred_hidden(const PredictLaunc
     }
     __syncthreads();
 
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int steps = d / (kWarp * N) / p.splits;  // 16-byte vectors per lane per piece
-    const int seg = steps * kWarp * N;
-    const int total = p.r * p.splits;
-    for (int piece = blockIdx.x * kPredWarps + warp; piece < total; piece += gridDim.x * kPredWarps) {
+    bool loaded = true;  // v holds the first vectors of this piece
+    for (; piece < total; piece += gridDim.x * kPredWarps) {
         const int sp = piece / p.r, row = piece - sp * p.r;
-        const T* wrow = static_cast<const T*>(p.w1) + (size_t)row * d + (size_t)sp * seg + lane * N;
+        const T* wrow = wrow_of(piece);
         const float* xb = xs + (size_t)sp * seg + lane * N;
         float acc[NB];
 #pragma unroll
         for (int t = 0; t < NB; ++t) acc[t] = 0.0f;
         for (int s0 = 0; s0 < steps; s0 += 8) {
-            uint4 v[8];
+            if (!loaded) {
 #pragma unroll
-            for (int u = 0; u < 8; ++u)
-                v[u] = s0 + u < steps ? ld_stream(wrow + (size_t)(s0 + u) * kWarp * N) : make_uint4(0u, 0u, 0u, 0u);
+                for (int u = 0; u < 8; ++u)
+                    v[u] = s0 + u < steps ? ld_stream(wrow + (size_t)(s0 + u) * kWarp * N)
+                                          : make_uint4(0u, 0u, 0u, 0u);
+            }
+            loaded = false;
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
                 if (s0 + u < steps) {
@@ -125,11 +143,28 @@ __device__ __forceinline__ unsigned order_key(float f) {
 template <typename T, int NB, int STEPS>
 __global__ void __launch_bounds__(kPredThreads) k_pred_score(const PredictLaunch p) {
     extern __shared__ __align__(16) float hs[];  // [NB][r]
-    pdl_wait();
-    pdl_launch_dependents();
     constexpr int N = Vec<T>::N;
     constexpr int RG = STEPS >= 8 ? 1 : 8 / STEPS;
     const int r = p.r, m = p.m;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int groups = (m + RG - 1) / RG;
+    uint4 v[RG][STEPS];
+    auto load = [&](int g) {
+        const int j0 = g * RG;
+#pragma unroll
+        for (int q = 0; q < RG; ++q)
+#pragma unroll
+            for (int s = 0; s < STEPS; ++s)
+                v[q][s] = j0 + q < m ? ld_stream(static_cast<const T*>(p.w2) + (size_t)(j0 + q) * r +
+                                                 s * kWarp * N + lane * N)
+                                     : make_uint4(0u, 0u, 0u, 0u);
+    };
+    // W2 does not depend on earlier kernels: this warp's first group of rows
+    // is loaded before the wait, while the hidden-layer kernel runs.
+    int g = blockIdx.x * kPredWarps + warp;
+    if (g < groups) load(g);
+    pdl_launch_dependents();
+    pdl_wait();
     for (int i = threadIdx.x; i < NB * r; i += blockDim.x) {
         const int t = i / r, j = i - t * r;
         float s = 0.0f;
@@ -141,18 +176,11 @@ __global__ void __launch_bounds__(kPredThreads) k_pred_score(const PredictLaunch
     }
     __syncthreads();
 
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int groups = (m + RG - 1) / RG;
-    for (int g = blockIdx.x * kPredWarps + warp; g < groups; g += gridDim.x * kPredWarps) {
+    bool loaded = true;
+    for (; g < groups; g += gridDim.x * kPredWarps) {
         const int j0 = g * RG;
-        uint4 v[RG][STEPS];
-#pragma unroll
-        for (int q = 0; q < RG; ++q)
-#pragma unroll
-            for (int s = 0; s < STEPS; ++s)
-                v[q][s] = j0 + q < m ? ld_stream(static_cast<const T*>(p.w2) + (size_t)(j0 + q) * r +
-                                                 s * kWarp * N + lane * N)
-                                     : make_uint4(0u, 0u, 0u, 0u);
+        if (!loaded) load(g);
+        loaded = false;
         float acc[RG][NB];
 #pragma unroll
         for (int q = 0; q < RG; ++q)
