@@ -82,7 +82,10 @@ def test_predict_matches_oracle(ts, dtype, r, B, K_frac):
     _check_list(lst, ref["scores"], K)
 
 
-@pytest.mark.parametrize("m,K", [(1, 1), (5, 3), (1000, 999), (4097, 410), (33, 32)])
+# 16384 fills the single-CTA register select exactly (16 keys per thread);
+# 16385 and 20000 take the radix select over keys in shared memory
+@pytest.mark.parametrize("m,K", [(1, 1), (5, 3), (1000, 999), (4097, 410), (33, 32), (16384, 1638),
+                                 (16385, 1639), (20000, 3000)])
 def test_predict_ragged_sizes(ts, m, K):
     d, r, B = 256, 256, 2
     L, P, x = _inputs(d, r, m, B, torch.bfloat16, seed=1100 + m)
@@ -107,6 +110,20 @@ def test_predict_ties_go_to_the_lower_id(ts):
         # each tie pair (j, j+256) keeps j before j+256
         s = set(lst.tolist())
         assert all((j - 256) in s for j in s if j >= 256), f"K={K}: a higher twin kept without its lower one"
+
+
+@pytest.mark.parametrize("m", [3584, 14336, 20000])
+def test_predict_all_scores_equal(ts, m):
+    """W2 = 0 makes every score exactly 0: all keys tie (one histogram bin holds
+    them all), so the list is the K lowest ids."""
+    d, r, B = 256, 256, 1
+    L, P, x = _inputs(d, r, m, B, torch.bfloat16, seed=1250 + m)
+    w2 = torch.zeros_like(P.w2)
+    dev = torch.device("cuda")
+    pred = ts.Predictor(P.w1.to(dev), w2.to(dev), max_batch=B)
+    for K in (1, m // 10, m - 1, m):
+        lst = pred.predict(x.to(dev), K).cpu().numpy()
+        assert np.array_equal(lst, np.arange(K)), f"m={m} K={K}"
 
 
 def test_predict_full_size_mistral(ts):
