@@ -251,7 +251,11 @@ ts_status ts_moe_get_error(ts_moe* h, cudaStream_t stream);
  *   w1, w2     device [r][d] and [m][r], row-major (borrowed, 16-byte aligned)
  *   max_batch  largest batch of a prediction, 1..8
  * Scores accumulate in fp32. Returns TS_ERR_UNSUPPORTED for sizes without a
- * kernel, TS_ERR_OOM if scratch cannot be allocated.
+ * kernel, TS_ERR_OOM if scratch cannot be allocated. The handle owns its
+ * scratch (hidden-layer partials, per-neuron keys and a histogram of the
+ * keys), which serves one prediction at a time: predictions with the same
+ * handle must not overlap on the GPU (use one stream, or one handle per
+ * stream).
  */
 ts_status ts_predictor_create(ts_predictor** out, int d, int r, int m, ts_dtype dtype, const void* w1,
                               const void* w2, int max_batch);
