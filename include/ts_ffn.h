@@ -52,11 +52,14 @@ typedef enum {
 /*
  * Weight storage. TS_F32 and TS_BF16 rows hold d elements. TS_INT4 rows (the
  * weight-only 4-bit storage of the paper's INT4 models, Tables 7-9) hold d/2
- * bytes of 4-bit codes -- element i in byte i/2, the low nibble for even i --
- * followed by d/32 little-endian IEEE binary16 scales, one per group of 32
- * consecutive elements: weight i = scale[i/32] * (code[i] - 8). An INT4 row
- * is 9d/16 bytes and needs d to be a multiple of 256; its activations x are
- * bf16.
+ * bytes of 4-bit codes followed by d/32 little-endian IEEE binary16 scales,
+ * one per group of 32 consecutive elements: weight i = scale[i/32] *
+ * (code[i] - 8). Group G's codes are the 16 bytes at offset 16G, read as four
+ * little-endian 32-bit words w0..w3; element 8s + 2t + h of the group
+ * (s, t in 0..3, h in 0..1) is nibble s + 4h of word t, i.e. bits
+ * [4(s + 4h), 4(s + 4h) + 4) of w_t (the order in which one tensor-core lane
+ * consumes them). An INT4 row is 9d/16 bytes and needs d to be a multiple of
+ * 256; its activations x are bf16.
  */
 typedef enum { TS_F32 = 0, TS_BF16 = 1, TS_INT4 = 2 } ts_dtype;
 
@@ -105,7 +108,7 @@ ts_status ts_ffn_forward(ts_ffn* h, const void* x, int batch, float* y, cudaStre
 
 /*
  * y = (Combined(x) * Mask(x)) W_down with the top-k magnitude mask of Eq. 3
- * and Eq. 4 (Sec. 5): per token, Mask keeps the `keep` neurons with the
+ * and Eq. 4 (Sec. 3.2): per token, Mask keeps the `keep` neurons with the
  * largest |Combined| = max(0, g) max(0, u) (Eq. 2), a lower neuron index
  * winning a tie; the others contribute 0.
  *   x, batch, y, stream   as ts_ffn_forward (no predictor list)
@@ -173,9 +176,11 @@ ts_status ts_ffn_set_test_stall(ts_ffn* h, int on);
 /*
  * One FFN forward with no handle and no device allocation. The paper has no
  * counterpart: this is a calling convention, not part of the method. It
- * computes exactly what ts_ffn_forward computes (Eq. 1 + Eq. 2; active_idx
- * as there, for the predictor-driven mode of Sec. 7) with the same kernels,
- * for callers that cannot allocate device memory when they run the FFN.
+ * computes exactly what ts_ffn_forward computes, with the same kernels, for
+ * callers that cannot allocate device memory when they run the FFN (a memory
+ * pool that is full or must not grow, code that must not take the implicit
+ * device synchronisation of cudaFree, a plain C caller with nowhere to keep
+ * a handle).
  *   d, m, wdtype, w_gate, w_up, w_down   as ts_ffn_create (borrowed for the call)
  *   x, batch, y, stream, active_idx, n_active   as ts_ffn_forward
  * Scratch: a fixed array of the library's static device memory (~0.8 MB per
@@ -184,7 +189,9 @@ ts_status ts_ffn_set_test_stall(ts_ffn* h, int on);
  * allocated or freed by this call.
  * Set-up: the first call on a device (that device current) looks up the
  * scratch address and sets kernel attributes; make that first call before
- * any stream capture on the device.
+ * any stream capture on the device. Each call compares the current context
+ * with the one the set-up was made in and repeats the set-up when the
+ * context was recreated (e.g. after cudaDeviceReset).
  * Concurrency: all calls on a device share the one scratch, so calls whose
  * executions overlap (other streams, unordered host threads) race; the
  * caller serialises them.

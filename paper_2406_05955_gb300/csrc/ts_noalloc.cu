@@ -9,8 +9,9 @@
 // ts_ffn_create; here the scratch of the two kernels instead lives in one
 // fixed-size array of the library's own static device memory, which exists
 // as soon as the module is loaded on a device. Its address is looked up once
-// per device with cudaGetSymbolAddress and then handed to the same gate+up
-// and down kernels the handle API launches.
+// per device context with cudaGetSymbolAddress (again if the context is
+// recreated) and then handed to the same gate+up and down kernels the handle
+// API launches.
 //
 // What the scratch holds and what must start at zero: c values
 // (kMaxPass x m fp32), per-token gate/both bitmaps (batch x nbytes each),
@@ -24,6 +25,7 @@
 // Concurrency: every call on a device uses the same scratch, so calls whose
 // executions overlap (different streams, different host threads without
 // ordering) race on it. The caller serialises them.
+#include <cuda.h>
 #include <stdint.h>
 #include <string.h>
 
@@ -57,10 +59,47 @@ constexpr int kMaxDevices = 64;
 
 struct NoAllocDevice {
     bool ready = false;
+    unsigned long long ctx_id = 0;  // the context the set-up below belongs to
     char* scratch = nullptr;
     int num_sms = 1;
     int optin_smem = 48 * 1024;
 };
+
+// The driver's context queries, reached through the runtime so that the
+// library does not link libcuda itself.
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+
+// Unique id of the current context (0 if none is current or the query fails).
+// A context that was destroyed and created again (cudaDeviceReset, or a
+// primary context released and retained anew) gets a new id, and the set-up
+// of the old one -- the scratch address, the kernels' shared-memory
+// attributes -- no longer holds.
+unsigned long long current_ctx_id() {
+    static CtxGetCurrentFn get_current = nullptr;
+    static CtxGetIdFn get_id = nullptr;
+    static bool looked_up = false;
+    if (!looked_up) {
+        void* f0 = nullptr;
+        void* f1 = nullptr;
+        cudaDriverEntryPointQueryResult q0 = cudaDriverEntryPointSymbolNotFound, q1 = q0;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f0, 12000, cudaEnableDefault, &q0) ==
+                cudaSuccess &&
+            q0 == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<CtxGetCurrentFn>(f0);
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f1, 12000, cudaEnableDefault, &q1) == cudaSuccess &&
+            q1 == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<CtxGetIdFn>(f1);
+        cudaGetLastError();
+        looked_up = true;
+    }
+    if (get_current == nullptr || get_id == nullptr) return 0;
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return 0;
+    if (get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
 
 std::mutex g_setup_mu;
 NoAllocDevice g_dev[kMaxDevices];
@@ -72,20 +111,25 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];
 
 namespace {
 
-// First call on a device (with that device current): find the scratch,
-// read the device facts and set the kernels' shared-memory attributes.
+// First call on a device (with that device current), and the first call
+// after that device's context was recreated: find the scratch, read the
+// device facts and set the kernels' shared-memory attributes.
 ts_status setup_device(NoAllocDevice** out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return TS_ERR_CUDA;
     if (dev < 0 || dev >= kMaxDevices) return TS_ERR_UNSUPPORTED;
     std::lock_guard<std::mutex> lock(g_setup_mu);
     NoAllocDevice& nd = g_dev[dev];
-    if (!nd.ready) {
+    const unsigned long long id = current_ctx_id();
+    if (!nd.ready || id == 0 || id != nd.ctx_id) {
+        nd.ready = false;
         void* p = nullptr;
+        // also creates the device's primary context if none is current yet
         if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) {
             cudaGetLastError();
             return TS_ERR_CUDA;
         }
+        nd.ctx_id = current_ctx_id();
         if (cudaDeviceGetAttribute(&nd.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
             cudaDeviceGetAttribute(&nd.optin_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
                 cudaSuccess)

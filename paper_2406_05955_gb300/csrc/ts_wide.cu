@@ -15,7 +15,7 @@
 //                both-active rows p of c_t,p W_down[row p][:] (Eq. 1);
 //   k_wide_reduce y_t = sum over slices s in order (or h_t += y_t).
 // All products are mma.sync m16n8k16 (bf16 in, fp32 accumulate) on tiles
-// staged by 16-byte cp.async through a 4-stage shared-memory pipeline; row
+// staged by 16-byte cp.async through a kStages-deep shared-memory pipeline; row
 // tiles are gathered by index, so the sparsity of the union still skips rows.
 #include "ts_kernels.cuh"
 #include "ts_wide.h"

@@ -178,3 +178,30 @@ def test_int4_pins_reject_planted_mistakes(mistake):
 
 def test_int4_planted_mistake_control():
     test_int4_pins_reject_planted_mistakes(None)
+
+
+def test_header_packing_text_matches_quantize_int4():
+    """Pack INT4 rows exactly as the public header describes them and compare
+    the bytes with the generator's quantizer (the format the library reads):
+    group G's codes are the 16 bytes at 16G, four little-endian 32-bit words;
+    element 8s + 2t + h is nibble s + 4h of word t; then d/32 binary16 scales."""
+    rng = np.random.default_rng(11)
+    m, d = 3, 256
+    w = torch.from_numpy(rng.standard_normal((m, d)).astype(np.float32))
+    got = wl.quantize_int4(w).numpy()
+    wf = w.numpy().reshape(m, d // 32, 32)
+    scale = (np.abs(wf).max(-1) / 7.0).astype(np.float16)
+    scale[scale == 0] = 1
+    code = np.clip(np.round(wf / scale.astype(np.float32)[..., None]), -8, 7).astype(np.int64) + 8
+    want = np.zeros((m, d // 2 + d // 16), dtype=np.uint8)
+    for j in range(m):
+        for G in range(d // 32):
+            words = [0, 0, 0, 0]
+            for e in range(32):
+                s, t, h = e // 8, (e % 8) // 2, e % 2
+                words[t] |= int(code[j, G, e]) << (4 * (s + 4 * h))
+            for t in range(4):
+                for b in range(4):
+                    want[j, 16 * G + 4 * t + b] = (words[t] >> (8 * b)) & 0xFF
+        want[j, d // 2:] = np.frombuffer(scale[j].tobytes(), dtype=np.uint8)
+    np.testing.assert_array_equal(got, want)
