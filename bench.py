@@ -3,7 +3,12 @@
 One step = one decode token (batch 1) through all 32 FFN layers of the
 pre-norm residual stack (d=4096, m=14336, bf16 weights, ~10% combined dReLU
 activation), replayed from one CUDA graph. Weights (11.3 GB) exceed L2, so no
-flush is needed between steps. Prints one JSON line (rank 0).
+flush is needed between steps. The K timed steps form one region; the region
+is repeated (at least 3 times, enough to cover half a second) and the median
+region is reported. Prints one JSON line (rank 0). By default that line also
+carries, under "other_configs", the fp32 single FFN, the predictor-driven mode
+on the same 32 layers, the Mixtral-shaped MoE stack at batch 1 and 8, and the
+batch x activation sweep next to dense cuBLAS (--headline-only skips them).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                   [--workload stack|predictor|moe|sweep] [--batch B]
@@ -23,6 +28,7 @@ from __future__ import annotations
 import argparse
 import hashlib
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -48,9 +54,9 @@ NOMINAL_HBM_GBS = 7900.0
 # kernel sources they were taken on: once those change, the figures no longer
 # describe the kernels and are reported as null.
 KERNEL_SOURCES = ("paper_2406_05955_gb300/csrc/ts_gate_up.cu", "paper_2406_05955_gb300/csrc/ts_kernels.cuh")
-NCU_TRAFFIC = {"bytes": {"bf16": 164.22e6, "int4": 45.72e6},
+NCU_TRAFFIC = {"bytes": {"bf16": 164.48e6, "int4": 45.72e6},
                "sources": KERNEL_SOURCES,
-               "sha256": "360fb139726ef231f2f86638f86309a2f558dcc3bb4e28f3c5f6f27a13addba3"}
+               "sha256": "4f9a9d2a4347a69c4ee95e4a48d45d2b27ca90afbce485839545cd43258744db"}
 
 
 def kernel_sources_sha256(paths) -> str:
@@ -243,21 +249,52 @@ def time_graph(graph, stream, steps: int) -> float:
     return s.elapsed_time(e) / 1e3
 
 
-def time_kernel_gate_up(ts, ffns, x, stream, lists, reps: int) -> float:
-    """Average duration of one gate+up launch (the dominant kernel), CUDA events on its stream."""
-    for f_i, f in enumerate(ffns):
-        f.gate_up(x, active_idx=None if lists is None else lists[f_i], stream=stream)
+MIN_TIMED_S = 0.5  # the repeats of a timed region cover at least this long, so the clock sampler sees the load
+
+
+def time_repeats(graph, stream, steps: int, dist, min_total_s: float = MIN_TIMED_S):
+    """Time ``steps`` replays R >= 3 times, each region bracketed by a barrier and a
+    synchronize, R large enough that the regions cover ``min_total_s``.
+    Returns (per-region seconds, max over ranks; clocks sampled meanwhile)."""
+    dist.barrier()
     torch.cuda.synchronize()
-    evs = []
+    probe = time_graph(graph, stream, steps)
+    reps = int(max(3, min(500, math.ceil(min_total_s / max(probe, 1e-6)))))
+    reps = int(dist.max(float(reps)))
+    clocks = ClockSampler(dist.local)
+    clocks.start()
+    time.sleep(0.3)
+    times = []
     for _ in range(reps):
+        dist.barrier()
+        torch.cuda.synchronize()
+        el = time_graph(graph, stream, steps)
+        torch.cuda.synchronize()
+        dist.barrier()
+        times.append(dist.max(el))
+    return times, clocks.stop()
+
+
+def time_kernel_gate_up(ts, ffns, x, stream, lists, reps: int = 20) -> float:
+    """Average duration of one gate+up launch (the dominant kernel) launched
+    back to back, one per layer, the way the stack runs it (programmatic
+    dependent launch between consecutive launches): CUDA events on its stream
+    around ``reps`` passes over the layers, divided by the launches. The host
+    enqueues a launch in a few microseconds, well ahead of the ~35 us kernels."""
+    def body():
         for f_i, f in enumerate(ffns):
-            s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            s.record(stream)
             f.gate_up(x, active_idx=None if lists is None else lists[f_i], stream=stream)
-            e.record(stream)
-            evs.append((s, e))
+
+    for _ in range(2):
+        body()
     torch.cuda.synchronize()
-    return statistics.mean(s.elapsed_time(e) for s, e in evs) / 1e3
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record(stream)
+    for _ in range(reps):
+        body()
+    e.record(stream)
+    e.synchronize()
+    return s.elapsed_time(e) / 1e3 / (reps * len(ffns))
 
 
 def dense_cublas_tokens_per_s(layers, batch, dev, steps=10) -> float:
@@ -295,35 +332,181 @@ def dense_cublas_tokens_per_s(layers, batch, dev, steps=10) -> float:
     return batch * steps / (s.elapsed_time(e) / 1e3)
 
 
-def cpu_baseline(layers, lists, batch, n_layers_total, budget_s=12.0) -> dict:
-    """The oracle as it stands, on the host cores, over a bounded sample of layers."""
+def cpu_baseline(layers, lists, batch, n_layers_total, budget_s=12.0, budget_1t_s=6.0) -> dict:
+    """The oracle as it stands, on the host cores, over a bounded sample of
+    layers: with every core (OpenMP over independent outputs), then with one
+    thread (reported beside it)."""
     import oracle
 
     host = [(oracle.as_array(L.w_gate), oracle.as_array(L.w_up), oracle.as_array(L.w_down))
             for L in layers[:2]]
     hl = None if lists is None else [x.cpu().numpy() for x in lists[:2]]
-    rng = np.random.default_rng(0)
-    h = rng.standard_normal((batch, layers[0].d)).astype(np.float32)
-    done = 0
-    t0 = time.perf_counter()
-    while True:
-        i = done % len(host)
-        x = oracle.rmsnorm(h, oracle.BF16)
-        r = oracle.ffn(x, *host[i], rows=None if hl is None else hl[i])
-        h = (h + r["y"]).astype(np.float32)
-        done += 1
-        el = time.perf_counter() - t0
-        if el >= budget_s or done >= 400:
-            break
+    cores = oracle.max_threads()
+
+    def sample(threads: int, budget: float):
+        rng = np.random.default_rng(0)
+        h = rng.standard_normal((batch, layers[0].d)).astype(np.float32)
+        done = 0
+        t0 = time.perf_counter()
+        while True:
+            i = done % len(host)
+            x = oracle.rmsnorm(h, oracle.BF16)
+            r = oracle.ffn(x, *host[i], rows=None if hl is None else hl[i], threads=threads)
+            h = (h + r["y"]).astype(np.float32)
+            done += 1
+            el = time.perf_counter() - t0
+            if el >= budget or done >= 400:
+                return done, el
+
+    done, el = sample(cores, budget_s)
+    done1, el1 = sample(1, budget_1t_s)
+    oracle.ffn(*([np.zeros((1, 1), np.float32)] * 4), threads=cores)  # restore the thread count
     value = batch * done / n_layers_total / el
-    return {"value": value, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+    return {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": f"{done} layer evaluations (cycling over 2 of the {n_layers_total} layers, batch {batch}) "
-                      f"in {el:.1f} s, scaled to full {n_layers_total}-layer tokens"}
+                      f"in {el:.1f} s, scaled to full {n_layers_total}-layer tokens",
+            "single_thread": {"value": batch * done1 / n_layers_total / el1, "unit": UNIT, "cores": 1,
+                              "sample": f"{done1} layer evaluations in {el1:.1f} s, one OpenMP thread"}}
 
 
 # ---------------------------------------------------------------------------
 # arms
 # ---------------------------------------------------------------------------
+def predictor_line(ts, wl, ffns, layers, h0, stream, args, dist) -> dict:
+    """Predictor-driven mode (Sec. 7) on the given 32 layers at batch 1: per
+    layer a sorted list of 1434 neurons drawn with Zipf(1.1) weights over
+    hotness; gate, up and down touch only listed rows."""
+    name = "mistral7b-ffn-stack-bf16-predictor"
+    cfg = wl.WORKLOADS[name]
+    dev = h0.device
+    lists = [wl.predictor_list(L.offsets, cfg["list_len"], zipf_s=cfg["zipf_s"],
+                               seed=wl.layer_seed(cfg["seed"], l) + 7).to(dev) for l, L in enumerate(layers)]
+    h = h0.clone()
+    graph = ts.Graph.stack(ffns, h, active_idx=lists)
+    for _ in range(args.warmup):
+        graph.launch(stream)
+    torch.cuda.synchronize()
+    times, clk = time_repeats(graph, stream, args.steps, dist)
+    t = statistics.median(times)
+    nb = needed_bytes_stack(ffns, lists)
+    peaks = load_peaks()
+    step_s = t / args.steps
+    graph.close()
+    return {"workload": name, "value": whole_job_value(1, args.steps, dist.world, t), "unit": UNIT,
+            "ms_per_step": step_s * 1e3, "timed_regions": len(times),
+            "list_len": cfg["list_len"],
+            "needed_bytes_roofline": {"bytes_per_token": nb["gate_up"] + nb["down"],
+                                      "achieved_gbs": (nb["gate_up"] + nb["down"]) / step_s / 1e9,
+                                      "frac_of_measured": (nb["gate_up"] + nb["down"]) / step_s / 1e9 / peaks["hbm_gbs"]},
+            "clocks": clk}
+
+
+def fp32_small_line(ts, wl, dev, args, dist) -> dict:
+    """The fp32 single-FFN configuration (d=512, m=1408): 16 decode tokens one
+    at a time through one FFN, replayed from a graph. Its 4 MB of weights sit
+    in L2, so it is reported for speed only, not against the HBM roofline."""
+    name = "drelu-ffn-fp32-d512-m1408"
+    cfg = wl.WORKLOADS[name]
+    d, m, n_tok = cfg["d"], cfg["m"], cfg["n_tokens"]
+    L = wl.ffn_layer(d, m, mu=cfg["mu"], dtype=torch.float32, seed=cfg["seed"], device=dev)
+    f = ts.Ffn(L.w_gate, L.w_up, L.w_down, max_batch=1)
+    xs = wl.tokens(n_tok, d, dtype=torch.float32, seed=cfg["seed"] + 1, device=dev)
+    ys = torch.empty(n_tok, d, dtype=torch.float32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def body():
+        for t in range(n_tok):
+            f.forward(xs[t:t + 1], y=ys[t:t + 1], stream=stream)
+
+    with torch.cuda.stream(stream):
+        body()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        body()
+    calls = _Calls(lambda st: g.replay())
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            g.replay()
+        torch.cuda.synchronize()
+        times, clk = time_repeats(calls, stream, args.steps, dist)
+    t = statistics.median(times)
+    del g
+    f.close()
+    return {"workload": name, "value": whole_job_value(n_tok, args.steps, dist.world, t), "unit": UNIT,
+            "us_per_token": t / (args.steps * n_tok) * 1e6, "timed_regions": len(times),
+            "note": "L2-resident (4 MB of weights): a correctness configuration, no HBM roofline", "clocks": clk}
+
+
+def moe_lines(ts, wl, dev, args, dist, batches, int4: bool = False) -> list:
+    """32-layer Mixtral-shaped MoE stack (router + top-2 of 8 sparse experts
+    per layer), one timed line per batch size; the weights are drawn once."""
+    name = "mixtral47b-moe-stack-int4-top2" if int4 else "mixtral47b-moe-stack-bf16-top2"
+    cfg = wl.WORKLOADS[name]
+    d, m, E, k = cfg["d"], cfg["m"], cfg["experts"], cfg["top_k"]
+    n_layers = args.layers or cfg["layers"]
+    max_b = max(batches)
+    experts, moes = [], []
+    for l in range(n_layers):
+        if int4:
+            ex = [wl.ffn_layer_int4(d, m, activation=cfg["activation"], seed=wl.layer_seed(cfg["seed"], l, e),
+                                    device=dev) for e in range(E)]
+        else:
+            ex = [wl.ffn_layer(d, m, activation=cfg["activation"], dtype=torch.bfloat16,
+                               seed=wl.layer_seed(cfg["seed"], l, e), device=dev) for e in range(E)]
+        ffns = [ts.Ffn(L.w_gate, L.w_up, L.w_down, max_batch=max_b) for L in ex]
+        wr = wl.router(E, d, seed=wl.layer_seed(cfg["seed"], l) + 99, device=dev)
+        experts.append((ex, ffns, wr))
+        moes.append(ts.Moe(wr, ffns, top_k=k, max_batch=max_b))
+    peaks = load_peaks()
+    out = []
+    for B in batches:
+        h0 = wl.residual(B, d, seed=cfg["seed"] - 1, device=dev)
+        h = h0.clone()
+        stream = torch.cuda.Stream(device=dev)
+        graph = ts.Graph.moe_stack(moes, h)
+        for _ in range(args.warmup):
+            graph.launch(stream)
+        torch.cuda.synchronize()
+        times, clk = time_repeats(graph, stream, args.steps, dist)
+        t = statistics.median(times)
+        # needed bytes of the last replay: per layer, every expert a token was routed to
+        graph.launch(stream)
+        torch.cuda.synchronize()
+        need = 0
+        for mo in moes:
+            sel, _ = mo.get_routing(B)
+            for e in sorted(set(sel.ravel().tolist())):
+                g, b = mo.get_active(e, -1)
+                need += (m + len(g) + len(b)) * row_bytes(mo.experts[e])
+        step_s = t / args.steps
+        out.append({"workload": name, "batch": B, "value": whole_job_value(B, args.steps, dist.world, t),
+                    "unit": UNIT, "ms_per_step": step_s * 1e3, "timed_regions": len(times),
+                    "config": {"d": d, "m": m, "experts": E, "top_k": k, "layers": n_layers,
+                               "activation": cfg["activation"],
+                               "weights_gb": round(E * 3 * m * row_bytes(experts[0][1][0]) * n_layers / 1e9, 1)},
+                    "needed_bytes_roofline": {"bytes_per_step": need, "achieved_gbs": need / step_s / 1e9,
+                                              "frac_of_measured": need / step_s / 1e9 / peaks["hbm_gbs"]},
+                    "gpu_launches": 3 * n_layers * args.steps * ((B + 7) // 8),
+                    "clocks": clk})
+        graph.close()
+    for mo in moes:
+        mo.close()
+    for _, ffns, _ in experts:
+        for f in ffns:
+            f.close()
+    del experts, moes
+    torch.cuda.empty_cache()
+    return out
+
+
+def _sweep_summary(r: dict) -> dict:
+    return {"batch": r["config"]["batch"], "activation": r["config"]["activation"], "value": r["value"],
+            "unit": r["unit"], "ms_per_step": r["ms_per_step"],
+            "frac_of_measured": r["needed_bytes_roofline"]["frac_of_measured"],
+            "dense_cublas": r["dense_cublas"]["value"], "speedup_vs_dense": r["speedup_vs_dense"]}
+
+
 def run_ours(args, dist: Dist) -> dict | None:
     import paper_2406_05955_gb300 as ts
     from paper_2406_05955_gb300 import workload as wl
@@ -343,44 +526,35 @@ def run_ours(args, dist: Dist) -> dict | None:
         graph.launch(stream)
     torch.cuda.synchronize()
 
-    # timed region: K graph replays, barrier + sync on both sides, clocks sampled
-    clocks = ClockSampler(dist.local)
-    dist.barrier()
-    torch.cuda.synchronize()
-    clocks.start()
-    time.sleep(0.3)
-    elapsed = time_graph(graph, stream, args.steps)
-    torch.cuda.synchronize()
-    dist.barrier()
-    clk = clocks.stop()
-    t_max = dist.max(elapsed)
+    # timed region: K graph replays, barrier + sync on both sides, clocks
+    # sampled; repeated (>= 3 regions) and the median region taken
+    times, clk = time_repeats(graph, stream, args.steps, dist)
+    t_max = statistics.median(times)
     value = whole_job_value(B, args.steps, dist.world, t_max)
 
-    # end-to-end through the public API with host buffers (pinned), copies inside the timed region
+    # end-to-end through the public API with host buffers (pinned), copies
+    # inside the timed region; as many regions as above, median
     h_host = torch.empty_like(h0, device="cpu").pin_memory()
     h_host.copy_(h0.cpu())
     out_host = torch.empty_like(h_host).pin_memory()
-    s_ev, e_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    dist.barrier()
-    torch.cuda.synchronize()
-    s_ev.record(stream)
+    with_copies = _Calls(lambda st: (h.copy_(h_host, non_blocking=True), graph.launch(st),
+                                     out_host.copy_(h, non_blocking=True)))
+    e2e_times = []
     with torch.cuda.stream(stream):
-        for _ in range(args.steps):
-            h.copy_(h_host, non_blocking=True)
-            graph.launch(stream)
-            out_host.copy_(h, non_blocking=True)
-    e_ev.record(stream)
-    e_ev.synchronize()
-    e2e_t = dist.max(s_ev.elapsed_time(e_ev) / 1e3)
+        for _ in range(len(times)):
+            dist.barrier()
+            torch.cuda.synchronize()
+            e2e_times.append(dist.max(time_graph(with_copies, stream, args.steps)))
+    e2e_t = statistics.median(e2e_times)
     e2e = {"value": B * args.steps * dist.world / e2e_t, "unit": UNIT,
            "h2d_bytes_per_step": h_host.numel() * 4, "d2h_bytes_per_step": out_host.numel() * 4}
 
-    # dominant kernel: gate+up, timed alone per layer
+    # dominant kernel: gate+up, one launch per layer replayed from a graph
     x = wl.tokens(B, cfg["d"], dtype=torch.bfloat16, seed=5, device=dev)  # bf16 activations (INT4 too)
     graph.launch(stream)
     torch.cuda.synchronize()
     nb = needed_bytes_stack(ffns, lists)
-    t_gate_up = time_kernel_gate_up(ts, ffns, x, stream, lists, reps=3)
+    t_gate_up = time_kernel_gate_up(ts, ffns, x, stream, lists)
     nb_x = needed_bytes_stack(ffns, lists)  # active sets of the x used in the kernel timing
     peaks = load_peaks()
     # passes of 1-2 tokens: the gate+up kernel also gathers the W_down rows
@@ -394,6 +568,9 @@ def run_ours(args, dist: Dist) -> dict | None:
         "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int4 weights, bf16 activations, fp32 accumulate" if int4 else "bf16",
         "data": "synthetic",
+        "timing": {"timed_regions": len(times), "statistic": "median over regions",
+                   "ms_per_step_min": min(times) / args.steps * 1e3,
+                   "ms_per_step_max": max(times) / args.steps * 1e3},
         "config": {"workload": stack_workload(args),
                    "d": cfg["d"], "m": cfg["m"], "layers": n_layers, "batch": B,
                    "activation": cfg["activation"], "weights_gb": round(3 * cfg["m"] * row_bytes(ffns[0]) * n_layers / 1e9, 2),
@@ -417,7 +594,9 @@ def run_ours(args, dist: Dist) -> dict | None:
                      "frac": achieved / peaks["hbm_gbs"], "peak_source": peaks["source"],
                      "traffic": None if predictor or B != 1 else ncu_traffic("int4" if int4 else "bf16"),
                      "bytes_per_launch": gate_up_bytes,
-                     "avg_launch_us": t_gate_up * 1e6},
+                     "avg_launch_us": t_gate_up * 1e6,
+                     "timed_as": f"{n_layers} gate+up launches (one per layer) back to back, 20 passes, "
+                                 "CUDA events on the launching stream"},
         "e2e": e2e,
         "gpu_launches": 2 * n_layers * args.steps * ((B + 7) // 8),
         "clocks": clk,
@@ -427,23 +606,27 @@ def run_ours(args, dist: Dist) -> dict | None:
                                   "what": "same weights, dense ReLU-gated FFN via torch.matmul (cuBLAS), graph-replayed"}
     if dist.rank == 0 and not args.no_cpu_baseline and not int4:
         result["cpu_baseline"] = cpu_baseline(layers, lists, B, n_layers)
+    if args.workload == "stack" and B == 1 and not args.headline_only:
+        # the predictor-driven mode on the same 32 layers (its lists favour hot neurons)
+        graph.close()
+        result["other_configs"] = {"predictor_mode": predictor_line(ts, wl, ffns, layers, h0, stream, args, dist)}
     for f in ffns:
         f.close()
     graph.close()
+    del layers, ffns
+    torch.cuda.empty_cache()
+    if args.workload == "stack" and B == 1 and not args.headline_only:
+        oc = result["other_configs"]
+        oc["fp32_single_ffn"] = fp32_small_line(ts, wl, dev, args, dist)
+        oc["moe_top2"] = moe_lines(ts, wl, dev, args, dist, batches=(1, 8))
+        oc["sweep"] = [_sweep_summary(r) for r in run_sweep(args, dist)]
     return result
 
 
 def _clocked_time(graph, stream, steps, dist):
-    """K graph replays between barriers with clocks sampled: (seconds max over ranks, clocks)."""
-    clocks = ClockSampler(dist.local)
-    dist.barrier()
-    torch.cuda.synchronize()
-    clocks.start()
-    time.sleep(0.3)
-    elapsed = time_graph(graph, stream, steps)
-    torch.cuda.synchronize()
-    dist.barrier()
-    return dist.max(elapsed), clocks.stop()
+    """Median over >= 3 timed regions of K replays (time_repeats): (seconds, clocks)."""
+    times, clk = time_repeats(graph, stream, steps, dist)
+    return statistics.median(times), clk
 
 
 class _Calls:
@@ -597,68 +780,23 @@ def run_prednet(args, dist: Dist) -> dict:
 
 
 def run_moe(args, dist: Dist) -> dict:
-    """32-layer Mixtral-shaped MoE stack (router + top-2 of 8 sparse experts per layer)."""
+    """32-layer Mixtral-shaped MoE stack (router + top-2 of 8 sparse experts per layer) at --batch."""
     import paper_2406_05955_gb300 as ts
     from paper_2406_05955_gb300 import workload as wl
 
-    name = "mixtral47b-moe-stack-int4-top2" if args.workload == "moe-int4" else "mixtral47b-moe-stack-bf16-top2"
-    cfg = wl.WORKLOADS[name]
-    int4 = cfg["dtype"] == "int4"
     dev = torch.device("cuda", dist.local)
     torch.cuda.set_device(dev)
-    B, d, m, E, k = args.batch, cfg["d"], cfg["m"], cfg["experts"], cfg["top_k"]
-    n_layers = args.layers or cfg["layers"]
-    experts, moes = [], []
-    for l in range(n_layers):
-        if int4:
-            ex = [wl.ffn_layer_int4(d, m, activation=cfg["activation"], seed=wl.layer_seed(cfg["seed"], l, e),
-                                    device=dev) for e in range(E)]
-        else:
-            ex = [wl.ffn_layer(d, m, activation=cfg["activation"], dtype=torch.bfloat16,
-                               seed=wl.layer_seed(cfg["seed"], l, e), device=dev) for e in range(E)]
-        ffns = [ts.Ffn(L.w_gate, L.w_up, L.w_down, max_batch=B) for L in ex]
-        wr = wl.router(E, d, seed=wl.layer_seed(cfg["seed"], l) + 99, device=dev)
-        experts.append((ex, ffns, wr))
-        moes.append(ts.Moe(wr, ffns, top_k=k, max_batch=B))
-    h0 = wl.residual(B, d, seed=cfg["seed"] - 1, device=dev)
-    h = h0.clone()
-    stream = torch.cuda.Stream(device=dev)
-    graph = ts.Graph.moe_stack(moes, h)
-    for _ in range(args.warmup):
-        graph.launch(stream)
-    torch.cuda.synchronize()
-    t_max, clk = _clocked_time(graph, stream, args.steps, dist)
-    value = whole_job_value(B, args.steps, dist.world, t_max)
-    # needed bytes of the last replay: per layer, every expert a token was routed to
-    graph.launch(stream)
-    torch.cuda.synchronize()
-    need = 0
-    for mo in moes:
-        sel, _ = mo.get_routing(B)
-        for e in sorted(set(sel.ravel().tolist())):
-            g, b = mo.get_active(e, -1)
-            need += (m + len(g) + len(b)) * row_bytes(mo.experts[e])
-    peaks = load_peaks()
-    step_s = t_max / args.steps
-    res = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "int4 weights, bf16 activations, fp32 accumulate" if int4 else "bf16",
-        "data": "synthetic",
-        "config": {"workload": name, "d": d, "m": m, "experts": E, "top_k": k, "layers": n_layers, "batch": B,
-                   "activation": cfg["activation"],
-                   "weights_gb": round(E * 3 * m * row_bytes(experts[0][1][0]) * n_layers / 1e9, 1),
-                   "l2": "no flush: the experts streamed per step exceed the 129 MB L2",
-                   "parallelism": f"replicas x{dist.world}"},
-        "needed_bytes_roofline": {"bytes_per_token": need / B, "achieved_gbs": need / step_s / 1e9,
-                                  "frac_of_measured": need / step_s / 1e9 / peaks["hbm_gbs"]},
-        "gpu_launches": 3 * n_layers * args.steps,
-        "clocks": clk,
-    }
-    for mo in moes:
-        mo.close()
-    graph.close()
-    return res
+    r = moe_lines(ts, wl, dev, args, dist, batches=(args.batch,), int4=args.workload == "moe-int4")[0]
+    int4 = args.workload == "moe-int4"
+    return {"metric": METRIC, "value": r["value"], "unit": UNIT, "n_gpus": dist.world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": r["ms_per_step"], "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None,
+            "dtype": "int4 weights, bf16 activations, fp32 accumulate" if int4 else "bf16", "data": "synthetic",
+            "config": dict(workload=r["workload"], batch=args.batch, **r["config"],
+                           l2="no flush: the experts streamed per step exceed the 129 MB L2",
+                           parallelism=f"replicas x{dist.world}"),
+            "needed_bytes_roofline": r["needed_bytes_roofline"], "gpu_launches": r["gpu_launches"],
+            "clocks": r["clocks"]}
 
 
 def run_sweep(args, dist: Dist) -> list:
@@ -686,7 +824,8 @@ def run_sweep(args, dist: Dist) -> list:
                 graph.launch(stream)
             torch.cuda.synchronize()
             steps = max(3, args.steps // max(1, B // 4))
-            t_max, clk = _clocked_time(graph, stream, steps, dist)
+            times, clk = time_repeats(graph, stream, steps, dist, min_total_s=0.2)
+            t_max = statistics.median(times)
             value = whole_job_value(B, steps, dist.world, t_max)
             nb = needed_bytes_stack(ffns, None)
             step_s = t_max / steps
@@ -768,6 +907,8 @@ def main():
                     help="fewer layers than the workload's 32 (profiling cases only; not a bench line)")
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--headline-only", action="store_true",
+                    help="default workload: skip the other configurations (fp32 FFN, predictor mode, MoE, sweep)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

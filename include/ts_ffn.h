@@ -306,6 +306,29 @@ ts_status ts_graph_capture_moe_stack(ts_graph** out, ts_moe* const* layers, int 
 ts_status ts_graph_capture_stack_predicted(ts_graph** out, ts_ffn* const* layers, ts_predictor* const* preds,
                                            int n_layers, float* h, int batch, const int* K,
                                            int32_t* const* lists);
+/*
+ * The same stack as ts_graph_capture_stack (Eq. 1 with the dReLU of Eq. 2 per
+ * layer, the stack glue between layers), fused into one persistent launch:
+ * every CTA (one per SM, all resident at once by a cooperative launch) runs
+ * each layer's gate+up phases and its share of the down projection, then the
+ * CTAs meet at a grid barrier, sum the partial down projections by column
+ * slices into h, meet again and go on with the next layer. No launch gaps
+ * between layers; one launch per replay, plus a memset that clears the
+ * barrier words.
+ *   layers, n_layers, h, batch, active_idx, n_active   as ts_graph_capture_stack
+ * Supported: bf16 layers of one width d, batch 1 or 2, the same grid for
+ * every layer; otherwise TS_ERR_UNSUPPORTED (capture the unfused stack then).
+ * The graph owns a small device table of the layers' parameters (allocated
+ * here, freed by ts_graph_destroy). Replays are bitwise identical to the
+ * unfused graph's only up to the fp32 summation order of the reduction (the
+ * partials are added in CTA order in both, in different groupings).
+ * Device-side errors (bad list entries, a barrier that waited past its
+ * bound: TS_ERR_TIMEOUT, after which the CTAs stop and h is undefined) are
+ * reported by ts_ffn_get_error on layers[0] (barriers) and on each layer
+ * (lists).
+ */
+ts_status ts_graph_capture_stack_fused(ts_graph** out, ts_ffn* const* layers, int n_layers, float* h,
+                                       int batch, const int32_t* const* active_idx, const int* n_active);
 ts_status ts_graph_launch(ts_graph* g, cudaStream_t stream);
 void ts_graph_destroy(ts_graph* g);
 

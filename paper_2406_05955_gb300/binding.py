@@ -52,6 +52,7 @@ SIGNATURES = {
     "ts_moe_get_active": (I, [P, P, I, I, P, IP, P, IP]),
     "ts_moe_get_error": (I, [P, P]),
     "ts_graph_capture_stack": (I, [PP, P, I, P, I, P, P]),
+    "ts_graph_capture_stack_fused": (I, [PP, P, I, P, I, P, P]),
     "ts_graph_capture_moe_stack": (I, [PP, P, I, P, I]),
     "ts_predictor_create": (I, [PP, I, I, I, I, P, P, I]),
     "ts_predictor_destroy": (None, [P]),
@@ -483,6 +484,19 @@ class Graph:
         g = ctypes.c_void_p()
         _check(lib().ts_graph_capture_stack(ctypes.byref(g), _addr(arr), len(layers), h.data_ptr(),
                                             h.shape[0], _addr(ptrs), _addr(ns)), "ts_graph_capture_stack")
+        return cls(g, (list(layers), h, keep))
+
+    @classmethod
+    def stack_fused(cls, layers, h: torch.Tensor, active_idx=None) -> "Graph":
+        """The stack as one persistent launch (ts_graph_capture_stack_fused);
+        raises TsError(TS_ERR_UNSUPPORTED) where it does not apply."""
+        _dev(h, "h")
+        arr = _handles(layers)
+        ptrs, ns, keep = _lists(active_idx, len(layers))
+        g = ctypes.c_void_p()
+        _check(lib().ts_graph_capture_stack_fused(ctypes.byref(g), _addr(arr), len(layers), h.data_ptr(),
+                                                  h.shape[0], _addr(ptrs), _addr(ns)),
+               "ts_graph_capture_stack_fused")
         return cls(g, (list(layers), h, keep))
 
     @classmethod

@@ -18,7 +18,8 @@ using namespace tsffn;
 namespace {
 
 constexpr size_t kAlign = 256;
-// rows of the next layer's W_gate each gate+up CTA prefetches into L2 (stack mode)
+// rows of the next layer's W_gate each gate+up CTA prefetches into L2 (stack
+// mode, passes of 4-8 tokens: the gathered down kernel issues them)
 constexpr int kPrefetchRows = 32;
 
 size_t align_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
@@ -151,6 +152,7 @@ struct ts_predictor {
 struct ts_graph {
     cudaGraph_t graph = nullptr;
     cudaGraphExec_t exec = nullptr;
+    void* mem = nullptr;  // device memory the captured kernels read (fused stack: layer table, barrier)
 };
 
 extern "C" {
@@ -404,7 +406,7 @@ ts_status read_status(unsigned* status_dev, cudaStream_t stream) {
 // rows (all, or the list). `next` is the following layer when it runs dense
 // (its first W_gate rows are then prefetched into L2), else nullptr.
 ts_status stack_layer(ts_ffn* h, const ts_ffn* next, float* hres, int batch, const int32_t* rows, int nr,
-                      cudaStream_t stream) {
+                      cudaStream_t stream, bool rows_ready) {
     if (use_wide(h, batch)) {
         WideLaunch L = wide_launch(h, batch, rows, nr);
         L.x = h->w_x;
@@ -420,6 +422,7 @@ ts_status stack_layer(ts_ffn* h, const ts_ffn* next, float* hres, int batch, con
     a.h = hres;
     a.norm_from_h = 1;
     a.residual_out = 1;
+    a.rows_ready = rows != nullptr && rows_ready ? 1 : 0;
     if (next != nullptr && batch <= kMaxPass && h->dt != TS_INT4) {
         a.next_wg = next->wg;
         a.next_n_rows = next->m;
@@ -530,8 +533,11 @@ ts_status ts_stack_forward(ts_ffn* const* layers, int n_layers, float* hres, int
     for (int l = 0; l < n_layers; ++l) {
         const int32_t* rows = active_idx ? active_idx[l] : nullptr;
         const bool next_dense = l + 1 < n_layers && !(active_idx && active_idx[l + 1]);
+        // a caller's list is in memory before the stack starts; from the
+        // second layer on, every kernel before the launch has finished with
+        // the first layer's wait, so the list may be read before waiting
         ts_status st = stack_layer(layers[l], next_dense ? layers[l + 1] : nullptr, hres, batch, rows,
-                                   rows ? n_active[l] : 0, stream);
+                                   rows ? n_active[l] : 0, stream, l > 0);
         if (st != TS_OK) return st;
     }
     return TS_OK;
@@ -887,7 +893,7 @@ ts_status ts_stack_forward_predicted(ts_ffn* const* layers, ts_predictor* const*
         PredictLaunch q = predict_launch(preds[l], batch, K[l], lists[l], nullptr);
         q.h = hres;
         ts_status st = cuda_status(launch_predict(q, elem_size(preds[l]->dt), stream, true));
-        if (st == TS_OK) st = stack_layer(h, nullptr, hres, batch, lists[l], K[l], stream);
+        if (st == TS_OK) st = stack_layer(h, nullptr, hres, batch, lists[l], K[l], stream, false);
         if (st != TS_OK) return st;
     }
     return TS_OK;
@@ -954,6 +960,82 @@ ts_status ts_graph_capture_stack_predicted(ts_graph** out, ts_ffn* const* layers
     });
 }
 
+ts_status ts_graph_capture_stack_fused(ts_graph** out, ts_ffn* const* layers, int n_layers, float* hres,
+                                       int batch, const int32_t* const* active_idx, const int* n_active) {
+    if (!out) return TS_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!layers || n_layers < 1 || !hres || batch < 1) return TS_ERR_INVALID_ARG;
+    if (((uintptr_t)hres & 15u) != 0) return TS_ERR_INVALID_ARG;
+    const ts_ffn* h0 = layers[0];
+    if (!h0) return TS_ERR_INVALID_ARG;
+    DeviceInfo dev;
+    ts_status st = device_info(&dev);
+    if (st != TS_OK) return st;
+    const int w = pow2_tokens(batch);
+    if (batch > kAccMaxTokens || h0->dt != TS_BF16) return TS_ERR_UNSUPPORTED;
+    const int grid = h0->grid[w];
+    for (int l = 0; l < n_layers; ++l) {
+        const ts_ffn* h = layers[l];
+        if (!h || h->d != h0->d || h->dt != h0->dt || batch > h->max_batch) return TS_ERR_INVALID_ARG;
+        if (h->grid[w] != grid || use_wide(h, batch)) return TS_ERR_UNSUPPORTED;
+        const int32_t* rows = active_idx ? active_idx[l] : nullptr;
+        if (rows && !n_active) return TS_ERR_INVALID_ARG;
+        st = check_list(h, rows, rows ? n_active[l] : 0);
+        if (st != TS_OK) return st;
+    }
+    if (!stack_fused_supported(h0->d, w, grid, dev.optin_smem)) return TS_ERR_UNSUPPORTED;
+
+    std::vector<FfnLaunch> table(n_layers);
+    for (int l = 0; l < n_layers; ++l) {
+        const int32_t* rows = active_idx ? active_idx[l] : nullptr;
+        FfnLaunch a = ffn_launch(layers[l], batch, rows, rows ? n_active[l] : 0);
+        a.h = hres;
+        a.norm_from_h = 1;
+        a.residual_out = 1;
+        a.tok0 = 0;
+        a.nt = batch;
+        a.bits_tok_base = 0;
+        a.partial_ctas = grid;
+        table[l] = a;
+    }
+    const size_t table_bytes = align_up(sizeof(FfnLaunch) * (size_t)n_layers);
+    void* mem = nullptr;
+    const size_t bar_bytes = align_up(sizeof(unsigned) * (size_t)stack_bar_words(grid));
+    if (cudaMalloc(&mem, table_bytes + bar_bytes) != cudaSuccess) {
+        cudaGetLastError();
+        return TS_ERR_OOM;
+    }
+    if (cudaMemcpy(mem, table.data(), sizeof(FfnLaunch) * (size_t)n_layers, cudaMemcpyHostToDevice) !=
+        cudaSuccess) {
+        cudaFree(mem);
+        return TS_ERR_CUDA;
+    }
+    StackLaunch S;
+    S.layers = static_cast<const FfnLaunch*>(mem);
+    S.n_layers = n_layers;
+    S.h = hres;
+    S.bar = reinterpret_cast<unsigned*>(static_cast<char*>(mem) + table_bytes);
+    S.status = h0->s.status;
+    ts_graph* g = nullptr;
+    st = capture(&g, [&](cudaStream_t s) {
+        // the barrier words and the abort flag start at zero on every replay
+        ts_status r = cuda_status(cudaMemsetAsync(S.bar, 0, bar_bytes, s));
+        if (r == TS_OK) r = cuda_status(launch_stack_fused(S, h0->d, w, grid, s));
+        return r;
+    });
+    if (st != TS_OK) {
+        cudaFree(mem);
+        return st;
+    }
+    g->mem = mem;
+    for (int l = 0; l < n_layers; ++l) {
+        const int32_t* rows = active_idx ? active_idx[l] : nullptr;
+        remember(layers[l], batch, rows, rows ? n_active[l] : 0);
+    }
+    *out = g;
+    return TS_OK;
+}
+
 ts_status ts_graph_launch(ts_graph* g, cudaStream_t stream) {
     if (!g || !g->exec) return TS_ERR_INVALID_ARG;
     return cuda_status(cudaGraphLaunch(g->exec, stream));
@@ -963,6 +1045,7 @@ void ts_graph_destroy(ts_graph* g) {
     if (!g) return;
     if (g->exec) cudaGraphExecDestroy(g->exec);
     if (g->graph) cudaGraphDestroy(g->graph);
+    if (g->mem) cudaFree(g->mem);
     delete g;
 }
 

@@ -228,6 +228,7 @@ constexpr int kRedCols = 64;
 constexpr int kRedThreads = 512;
 constexpr int kRedWarps = kRedThreads / kWarp;
 constexpr int kRedLanes = kRedCols / 4;  // lanes of a half-warp, a float4 each
+constexpr int kRedBatch = 6;  // partial blocks a half-warp has in flight
 
 template <int NT>
 __global__ void __launch_bounds__(kRedThreads) k_down_reduce(const FfnLaunch a) {
@@ -256,17 +257,32 @@ __global__ void __launch_bounds__(kRedThreads) k_down_reduce(const FfnLaunch a) 
 #pragma unroll
     for (int k = 0; k < NT; ++k) acc[k] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
     if (valid) {
+        // this half-warp's partial blocks b = warp * 2 + hw + i * 2 * kRedWarps:
+        // kRedBatch of them loaded at once, then added in the same order
         const size_t cta_stride = (size_t)a.partial_slots * d;
-        for (int b = warp * 2 + hw; b < a.partial_ctas; b += 2 * kRedWarps) {
-            const float* p = a.partial + (size_t)b * cta_stride + col;
+        constexpr int kStride = 2 * kRedWarps;
+        for (int b0 = warp * 2 + hw; b0 < a.partial_ctas; b0 += kRedBatch * kStride) {
+            float4 v[kRedBatch][NT];
 #pragma unroll
-            for (int k = 0; k < NT; ++k)
-                if (k < n_slots) {
-                    const float4 v = *reinterpret_cast<const float4*>(p + (size_t)k * d);
-                    acc[k].x += v.x;
-                    acc[k].y += v.y;
-                    acc[k].z += v.z;
-                    acc[k].w += v.w;
+            for (int i = 0; i < kRedBatch; ++i) {
+                const int b = b0 + i * kStride;
+                const float* p = a.partial + (size_t)b * cta_stride + col;
+#pragma unroll
+                for (int k = 0; k < NT; ++k)
+                    v[i][k] = (b < a.partial_ctas && k < n_slots) ? *reinterpret_cast<const float4*>(p + (size_t)k * d)
+                                                                  : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            }
+#pragma unroll
+            for (int i = 0; i < kRedBatch; ++i)
+                if (b0 + i * kStride < a.partial_ctas) {
+#pragma unroll
+                    for (int k = 0; k < NT; ++k)
+                        if (k < n_slots) {
+                            acc[k].x += v[i][k].x;
+                            acc[k].y += v[i][k].y;
+                            acc[k].z += v[i][k].z;
+                            acc[k].w += v[i][k].w;
+                        }
                 }
         }
     }

@@ -282,13 +282,15 @@ __device__ void finalize_chunk(const FfnLaunch& a, GateUpShared<NT>& sh, int cw,
 // them), all blocks of a group of rows in flight at once, and accumulates in
 // registers. A round after the first adds onto the stored partial, so the
 // order stays fixed and the result is bitwise reproducible.
+constexpr int kPartialLoads = 16;  // 16-byte W_down loads a lane has in flight in the down partial
+
 template <typename T, int NT, int NB>
 __device__ __forceinline__ void partial_blocks(const FfnLaunch& a, GateUpShared<NT>& sh, int n, int blk0,
                                                int bstride, float* pbase, bool accumulate, int lane) {
     constexpr int VEC = Vec<T>::N;
     constexpr int BLK = kWarp * VEC;
     constexpr int AT = NT;      // batch slots held (NT <= kAccMaxTokens)
-    constexpr int U = 16 / NB;  // rows per group: 16 loads in flight per lane
+    constexpr int U = kPartialLoads / NB;  // rows per group: kPartialLoads loads in flight per lane
     const int d = a.d;
     const int n_slots = a.route ? a.batch : a.nt;
     int col[NB];
@@ -1713,7 +1715,7 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(co
         for (int q = 0; q < kMaxLocal; ++q) sh.pd.ub[q] = 0;
         mbar_fence_init();
     }
-    const bool early = a.rows == nullptr && a.route == nullptr;
+    const bool early = (a.rows == nullptr || a.rows_ready) && a.route == nullptr;
     if (!early) pdl_wait();
     resolve_experts(a, sh.es);
     pdl_launch_dependents();
@@ -1749,6 +1751,201 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(co
     };
     consume_rows<T, NT>(a, sh, ring, xs, tab, ulist, rc, i0, i1, n_chunks, warp - 1, lane, stage);
     down_partial<T, NT>(a, sh, i0, i1, n_chunks, warp - 1, lane);
+}
+
+// ---------------------------------------------------------------------------
+// Fused layer stack: the per-layer chain of Eq. 1-2 for every layer of a
+// decode step inside one persistent launch.
+//
+// One CTA per SM, all co-resident (cooperative launch). Per layer, each CTA
+// runs the copy-by-consumer gate+up phases over its chunks and its share of
+// the down projection into its partial block, exactly as k_gate_up_rows;
+// then, instead of ending the kernel and launching the reduction:
+//   grid barrier -> CTA s sums the partial blocks of column slice s (32
+//   columns, blocks in CTA order) into the residual -> grid barrier -> the
+//   next layer stages rmsnorm(h).
+// A grid barrier is one atomic add per CTA on a word whose top bit flips
+// once every CTA has arrived; its wait is bounded (kGridWaitLimitNs), after
+// which the CTA records kStatusTimeout, raises the abort flag (so the others
+// stop at their next barrier instead of waiting out the limit) and returns.
+// (Measured alternatives: two-level arrival counters and per-CTA epoch words
+// polled by every CTA both made each layer slower.)
+// ---------------------------------------------------------------------------
+constexpr unsigned long long kGridWaitLimitNs = 4 * kWaitLimitNs;
+constexpr int kSliceCols = 32;  // columns a CTA reduces per slice (128 bytes of fp32)
+
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Grid barrier; consumer threads only (ctid in [0, cthreads)); false when
+// the stack must stop. Each CTA adds to one word: CTA 0 adds 2^31 - (grid -
+// 1), every other CTA 1, so the word's top bit flips exactly when the last
+// CTA arrives, whatever the order, and again at the next barrier. S.bar
+// (zero at launch): word 0 the barrier word, word 1 the abort flag.
+__device__ bool grid_barrier(const StackLaunch& S, int ctid, int cthreads, int* s_ok) {
+    named_bar_sync(1, cthreads);
+    if (ctid == 0) {
+        int ok = 1;
+        __threadfence();
+        const unsigned inc = blockIdx.x == 0 ? 0x80000000u - (gridDim.x - 1u) : 1u;
+        const unsigned old = atomicAdd(S.bar, inc);
+        const unsigned long long t0 = global_ns();
+        for (;;) {
+            if ((ld_acquire_u32(S.bar) ^ old) & 0x80000000u) break;
+            if (ld_acquire_u32(S.bar + 1) != 0u) {
+                ok = 0;
+                break;
+            }
+            if (global_ns() - t0 > kGridWaitLimitNs) {
+                atomicOr(S.status, kStatusTimeout);
+                atomicExch(S.bar + 1, 1u);
+                ok = 0;
+                break;
+            }
+        }
+        __threadfence();
+        *s_ok = ok;
+    }
+    named_bar_sync(1, cthreads);
+    return *s_ok != 0;
+}
+
+// h[t][cols of slice s] += sum over the partial blocks of partial[b][t][cols]
+// in the order of k_down_reduce, so that the fused stack gives the unfused
+// stack's bits: block group g (blocks g, g + 32, g + 64, ...) is summed in
+// ascending order, groups 2w and 2w + 1 are added, and those pair sums are
+// added for w = 0, 1, ... 15 onto 0. 256 consumer threads = 8 float4 columns
+// x 32 block groups.
+template <int NT>
+__device__ void reduce_slices(const FfnLaunch& a, float* h, int ctid, float4* red) {
+    const int d = a.d;
+    const int n_slices = (d + kSliceCols - 1) / kSliceCols;
+    const int q = ctid & 7;   // float4 column within the slice
+    const int gq = ctid >> 3; // block group: blocks gq, gq + 32, ...
+    const int nt = a.nt;
+    for (int sl = blockIdx.x; sl < n_slices; sl += gridDim.x) {
+        const int col = sl * kSliceCols + 4 * q;
+        const bool valid = col < d;
+        float4 acc[NT];
+#pragma unroll
+        for (int t = 0; t < NT; ++t) acc[t] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (valid) {
+            constexpr int kB = 6;  // blocks in flight per thread
+            for (int b0 = gq; b0 < a.partial_ctas; b0 += kB * 32) {
+                float4 v[kB][NT];
+#pragma unroll
+                for (int i = 0; i < kB; ++i) {
+                    const int b = b0 + i * 32;
+#pragma unroll
+                    for (int t = 0; t < NT; ++t)
+                        v[i][t] = (b < a.partial_ctas && t < nt)
+                                      ? __ldcg(reinterpret_cast<const float4*>(
+                                            a.partial + ((size_t)b * a.partial_slots + t) * d + col))
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+#pragma unroll
+                for (int i = 0; i < kB; ++i)
+#pragma unroll
+                    for (int t = 0; t < NT; ++t) {
+                        acc[t].x += v[i][t].x;
+                        acc[t].y += v[i][t].y;
+                        acc[t].z += v[i][t].z;
+                        acc[t].w += v[i][t].w;
+                    }
+            }
+        }
+#pragma unroll
+        for (int t = 0; t < NT; ++t) red[(gq * NT + t) * 8 + q] = acc[t];
+        named_bar_sync(1, GateUpWarps<NT>::C * kWarp);
+        if (ctid < 8 * NT) {
+            const int t = ctid >> 3, qq = ctid & 7;
+            const int c = sl * kSliceCols + 4 * qq;
+            if (t < nt && c < d) {
+                float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int w = 0; w < 16; ++w) {
+                    const float4 u = red[((2 * w) * NT + t) * 8 + qq];
+                    const float4 v = red[((2 * w + 1) * NT + t) * 8 + qq];
+                    sum.x += u.x + v.x;
+                    sum.y += u.y + v.y;
+                    sum.z += u.z + v.z;
+                    sum.w += u.w + v.w;
+                }
+                float4* hp = reinterpret_cast<float4*>(h + (size_t)t * d + c);
+                const float4 old = __ldcg(hp);
+                *hp = make_float4(old.x + sum.x, old.y + sum.y, old.z + sum.z, old.w + sum.w);
+            }
+        }
+        named_bar_sync(1, GateUpWarps<NT>::C * kWarp);
+    }
+}
+
+template <int NT>
+__global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_stack_rows(const StackLaunch S, const RowsCfg rc) {
+    using T = __nv_bfloat16;
+    constexpr int C = GateUpWarps<NT>::C;
+    __shared__ GateUpShared<NT> sh;
+    __shared__ FfnLaunch la;  // the current layer's parameters
+    __shared__ int s_ok;
+    extern __shared__ __align__(128) unsigned char dyn[];
+    float* xs = reinterpret_cast<float*>(dyn);
+    unsigned char* ring = dyn + (size_t)NT * rc.xs_stride * sizeof(float);
+    ChunkState<NT>* tab = reinterpret_cast<ChunkState<NT>*>(ring + (size_t)C * (rc.ahead + 1) * rc.slot_bytes);
+    unsigned short* ulist = reinterpret_cast<unsigned short*>(tab + kQ4Round);
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    constexpr int kWords = (int)(sizeof(FfnLaunch) / sizeof(unsigned));
+    static_assert(sizeof(FfnLaunch) % sizeof(unsigned) == 0, "FfnLaunch copies as words");
+
+    auto load_layer = [&](int l, int tid, int nthr) {
+        const unsigned* src = reinterpret_cast<const unsigned*>(S.layers + l);
+        unsigned* dst = reinterpret_cast<unsigned*>(&la);
+        for (int i = tid; i < kWords; i += nthr) dst[i] = src[i];
+    };
+    if (threadIdx.x == 0) {
+        mbar_init(&sh.never, 1);
+        mbar_fence_init();
+    }
+    load_layer(0, threadIdx.x, blockDim.x);
+    __syncthreads();
+    resolve_experts(la, sh.es);  // a single FFN with the same tokens in every layer
+    if (warp == 0) return;
+    const int ctid = threadIdx.x - kWarp;
+    const int cthreads = C * kWarp;
+
+    for (int l = 0; l < S.n_layers; ++l) {
+        if (l > 0) {
+            load_layer(l, ctid, cthreads);
+            named_bar_sync(1, cthreads);
+        }
+        if (ctid < kMaxLocal) sh.pd.ub[ctid] = 0;
+        const int n_chunks = (la.n_rows + kChunk - 1) / kChunk;
+        const int i0 = (int)((long long)n_chunks * blockIdx.x / gridDim.x);
+        const int i1 = (int)((long long)n_chunks * (blockIdx.x + 1) / gridDim.x);
+        auto stage = [&](auto&& first_rows) {
+            bool started = false;
+            auto once = [&]() {
+                if (!started) {
+                    started = true;
+                    first_rows();
+                }
+            };
+            for (int t = 0; t < la.nt; ++t) {
+                float* xrow = xs + (size_t)t * rc.xs_stride;
+                stage_act_row<T>(S.h + (size_t)t * la.d, nullptr, la.d, ctid, cthreads, sh.red,
+                                 [&](int i, float v) { xrow[xs_index<T>(i)] = v; }, once);
+            }
+            once();
+            named_bar_sync(1, cthreads);
+        };
+        consume_rows<T, NT>(la, sh, ring, xs, tab, ulist, rc, i0, i1, n_chunks, warp - 1, lane, stage);
+        down_partial<T, NT>(la, sh, i0, i1, n_chunks, warp - 1, lane);
+        if (!grid_barrier(S, ctid, cthreads, &s_ok)) return;
+        reduce_slices<NT>(la, S.h, ctid, reinterpret_cast<float4*>(ring));
+        if (!grid_barrier(S, ctid, cthreads, &s_ok)) return;
+    }
 }
 
 // Shared memory of the copy-by-consumer kernel: activations, the ring (as
@@ -1871,6 +2068,50 @@ static cudaError_t launch_rows_t(const FfnLaunch& a, int grid, cudaStream_t stre
     return cudaLaunchKernelEx(&lc, k_gate_up_rows<T, NT>, a, rc);
 }
 
+template <int NT>
+static cudaError_t launch_stack_t(const StackLaunch& S, int d, int grid, cudaStream_t stream) {
+    RowsCfg rc;
+    const size_t smem = rows_smem(2, d, NT, g_optin - kSmemMargin, &rc);
+    if (smem + kSmemMargin > (size_t)g_optin) return cudaErrorInvalidValue;
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(GateUpWarps<NT>::THREADS);
+    lc.dynamicSmemBytes = smem;
+    lc.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;  // every CTA resident at once: the grid barriers rely on it
+    attr[0].val.cooperative = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    return cudaLaunchKernelEx(&lc, k_stack_rows<NT>, S, rc);
+}
+
+int stack_bar_words(int) { return 2; }
+
+bool stack_fused_supported(int d, int nt, int grid, int optin_smem) {
+    if (nt < 1 || nt > kAccMaxTokens || grid < 1 || d < 1 || (d * 2) % 16 != 0) return false;
+    RowsCfg rc;
+    const size_t smem = rows_smem(2, d, nt, optin_smem - kSmemMargin, &rc);
+    if (smem + kSmemMargin > (size_t)optin_smem) return false;
+    int per_sm = 0, dev = 0, sms = 0;
+    const cudaError_t e = nt == 1 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+                                        &per_sm, k_stack_rows<1>, GateUpWarps<1>::THREADS, smem)
+                                  : cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+                                        &per_sm, k_stack_rows<2>, GateUpWarps<2>::THREADS, smem);
+    if (e != cudaSuccess || cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return per_sm >= 1 && grid <= per_sm * sms;
+}
+
+cudaError_t launch_stack_fused(const StackLaunch& S, int d, int nt, int grid, cudaStream_t stream) {
+    if (nt == 1) return launch_stack_t<1>(S, d, grid, stream);
+    if (nt == 2) return launch_stack_t<2>(S, d, grid, stream);
+    return cudaErrorInvalidValue;
+}
+
 // bf16 passes of 1-2 tokens take the copy-by-consumer kernel when its ring fits
 static bool use_rows(int wdtype, int d, int pass_tokens) {
     RowsCfg rc;
@@ -1899,6 +2140,8 @@ static cudaError_t prepare_t(int optin) {
 }
 
 cudaError_t prepare_gate_up(int optin_smem) {
+    static_assert(sizeof(GateUpShared<2>) + sizeof(FfnLaunch) + 64 < kSmemMargin,
+                  "static shared memory of the fused stack exceeds the margin");
     static_assert(sizeof(GateUpShared<8>) < kSmemMargin && sizeof(GateUpShared<4>) < kSmemMargin &&
                       sizeof(GateUpShared<2>) < kSmemMargin && sizeof(GateUpShared<1>) < kSmemMargin,
                   "static shared memory exceeds the margin");
@@ -1917,6 +2160,8 @@ cudaError_t prepare_gate_up(int optin_smem) {
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_rows<__nv_bfloat16, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_rows<__nv_bfloat16, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_stack_rows<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_stack_rows<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_q4w<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_q4w<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     return e;

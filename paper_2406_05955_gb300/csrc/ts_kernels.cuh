@@ -85,15 +85,32 @@ struct FfnLaunch {
     // gate+up CTA wait on a barrier nothing arrives at, so the bounded wait
     // runs out and the status word records kStatusTimeout.
     int test_stall;
+    // Nonzero when `rows` (the predictor list) was written before the
+    // kernels preceding this launch in the stream ran, so it may be read
+    // before waiting for them (stack layers after the first, with the
+    // caller's lists).
+    int rows_ready;
     // Stack mode: the next layer's W_gate (nullptr: none), its row count and
-    // its gate+up grid. The down-projection CTAs, before waiting for the
-    // gate+up kernel, prefetch into L2 the first prefetch_rows rows each
-    // next-layer gate+up CTA will stream, so HBM keeps working while this
-    // layer's up rows and down projection finish.
+    // its gate+up grid. The gathered down kernel (passes of 4-8 tokens),
+    // before waiting for the gate+up kernel, prefetches into L2 the first
+    // prefetch_rows rows each next-layer gate+up CTA will stream, so HBM keeps
+    // working while this layer's up rows and down projection finish.
     const void* next_wg;
     int next_n_rows;
     int next_grid;
     int prefetch_rows;
+};
+
+// The fused layer stack (passes of 1-2 tokens, bf16 rows, single FFNs): one
+// cooperative launch runs every layer's gate+up, down partial and reduction,
+// with grid barriers between the dependent steps instead of kernel
+// boundaries.
+struct StackLaunch {
+    const FfnLaunch* layers;  // device array [n_layers]; each layer's own scratch
+    int n_layers;
+    float* h;                 // [nt][d] residual, updated in place
+    unsigned* bar;            // zero before the launch: barrier counters and abort flag (stack_bar_words)
+    unsigned* status;         // barrier timeouts are recorded here
 };
 
 struct RouterLaunch {
@@ -346,7 +363,7 @@ __device__ __forceinline__ void stage_act_row(const float* __restrict__ h, const
 #pragma unroll
             for (int k = 0; k < kStageVec; ++k) {
                 const int q = g0 + ctid + k * cthreads;
-                v[k] = q < d4 ? *reinterpret_cast<const float4*>(h + 4 * (size_t)q) : make_float4(0.f, 0.f, 0.f, 0.f);
+                v[k] = q < d4 ? __ldcg(reinterpret_cast<const float4*>(h + 4 * (size_t)q)) : make_float4(0.f, 0.f, 0.f, 0.f);
             }
             if (g0 == 0) after_loads();
 #pragma unroll
@@ -371,7 +388,7 @@ __device__ __forceinline__ void stage_act_row(const float* __restrict__ h, const
             for (int k = 0; k < kStageVec; ++k) {
                 const int q = g0 + ctid + k * cthreads;
                 if (q < d4) {
-                    const float4 w = kept ? v[k] : *reinterpret_cast<const float4*>(h + 4 * (size_t)q);
+                    const float4 w = kept ? v[k] : __ldcg(reinterpret_cast<const float4*>(h + 4 * (size_t)q));
                     put(4 * q, norm(4 * q, w.x));
                     put(4 * q + 1, norm(4 * q + 1, w.y));
                     put(4 * q + 2, norm(4 * q + 2, w.z));
@@ -444,4 +461,11 @@ int gate_up_config(int wdtype, int d, int x_tokens, int optin_smem, int* slots, 
                    int* xs_stride, size_t* smem);
 // Whether INT4 rows of d weights can run passes of `pass_tokens` tokens.
 bool int4_supported(int d, int pass_tokens, int optin_smem);
+// The fused layer stack: whether a stack of bf16 layers of width d, passes of
+// nt tokens (1-2), can run as one cooperative launch of `grid` CTAs; and the
+// launch.
+bool stack_fused_supported(int d, int nt, int grid, int optin_smem);
+cudaError_t launch_stack_fused(const StackLaunch& S, int d, int nt, int grid, cudaStream_t stream);
+// 32-bit words of StackLaunch::bar for a grid of `grid` CTAs.
+int stack_bar_words(int grid);
 }  // namespace tsffn

@@ -23,7 +23,6 @@
 namespace tsffn {
 namespace {
 
-constexpr int kTileRows = 96;  // gate/up: weight rows per CTA
 constexpr int kTileK = 64;     // gate/up: K per pipeline stage (128 bytes of a row)
 constexpr int kStages = 6;
 // gate/up: 8 warps; warp w takes row tiles 3(w%4) .. 3(w%4)+2 over the K-steps
@@ -156,221 +155,321 @@ __device__ void bit_emit(const unsigned* words, int n_bits, const BitScan& b, in
 }
 
 // ---------------------------------------------------------------------------
-// gate / up: C[t][i] = x_t . W[row(i)] for a tile of 96 rows, all tokens
+// gate / up on the 5th-generation tensor cores: D[i][t] = W[row(i)] . x_t for
+// a tile of 128 weight rows (the MMA's M) and all tokens padded to 16 MT (N),
+// accumulated in tensor memory.
+//
+// Every thread copies its share of each K-stage (the 128 gathered weight rows
+// and the activations, 128 bytes of each per stage) with 16-byte cp.async
+// into a 128-byte-swizzled K-major tile; once a stage has landed everywhere,
+// thread 0 issues its four tcgen05.mma (K = 16 each) and a tcgen05.commit
+// that arrives on the stage's mbarrier when those MMAs have read the stage.
+// The stage is refilled kMmaLag k-blocks later (so the copies never wait on
+// the MMA just issued), keeping kStages - kMmaLag stages of copies in
+// flight. The accumulator (128 lanes x 16 MT fp32 columns) is read back with
+// tcgen05.ld.
 // ---------------------------------------------------------------------------
-struct GuSmem {
-    static constexpr int kX = kTokPad * kTileK * 2;     // 8 KB per stage
-    static constexpr int kW = kTileRows * kTileK * 2;   // 12 KB per stage
-    static constexpr int kStage = kX + kW;
-    static constexpr int kPipe = kStages * kStage;      // 80 KB
-    static constexpr int kOut = kTokPad * kTileRows * 4;  // 24 KB (aliases the pipeline)
-    static_assert(kOut <= kPipe, "the output tile aliases the pipeline buffers");
-    static constexpr int kBytes = kPipe;
+constexpr int kTcRows = 128;  // weight rows per tile: the MMA's M
+constexpr int kMmaLag = 2;    // a stage is refilled kMmaLag k-blocks after its MMAs were issued
+
+__device__ __forceinline__ void tc_alloc(uint32_t* dst, uint32_t ncols) {  // warp-wide
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(dst)), "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tc_relinquish() {  // warp-wide
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tc_dealloc(uint32_t taddr, uint32_t ncols) {  // warp-wide
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+// D (tensor memory) = A B^T (+ D when `accumulate`), one thread issues it
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                       uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// arrive once on `bar` when every tcgen05.mma this thread issued so far has completed
+__device__ __forceinline__ void tc_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_addr(bar))
+                 : "memory");
+}
+// 32 lanes x 16 fp32 columns: lane l of the warp gets the 16 columns of TMEM lane (taddr lane + l)
+__device__ __forceinline__ void tc_ld16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+// shared-memory descriptor of a K-major bf16 tile with 128-byte rows and the
+// 128-byte swizzle (8-row atoms of 1024 bytes, atom-aligned start)
+__device__ __forceinline__ uint64_t sdesc_k128(uint32_t saddr) {
+    uint64_t dsc = (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address, 16-byte units
+    dsc |= (uint64_t)1 << 16;                            // leading byte offset (not used by this layout)
+    dsc |= (uint64_t)(1024 >> 4) << 32;                  // stride byte offset: between 8-row atoms
+    dsc |= (uint64_t)1 << 46;                            // descriptor version
+    dsc |= (uint64_t)2 << 61;                            // 128-byte swizzle
+    return dsc;
+}
+// instruction descriptor: bf16 A and B (both K-major), fp32 D, shape M x N
+constexpr uint32_t idesc_bf16_f32(int M, int N) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+template <int MT>
+struct TcCfg {
+    static constexpr int NP = 16 * MT;                 // MMA N: tokens padded to 16
+    static constexpr int kA = kTcRows * 128;           // 16 KB of weight rows per stage
+    static constexpr int kB = NP * 128;                // activations per stage
+    static constexpr int kStage = kA + kB;
+    static constexpr int kStages = (192 * 1024) / kStage > 8 ? 8 : (192 * 1024) / kStage;
+    static constexpr int kBytes = kStages * kStage + 1024;  // + slack to align the tiles to 1024 bytes
+    static constexpr uint32_t kCols = NP <= 16 ? 32 : (NP <= 32 ? 64 : 128);  // tensor-memory columns: a power of 2, >= 2 N
+    static constexpr uint32_t kIdesc = idesc_bf16_f32(kTcRows, NP);
+    static_assert(NP % 16 == 0 && NP <= 256, "N of an M = 128 MMA");
 };
 
-// The tile's GEMM. rows_j[i] (shared) is the weight row of tile row i (-1: zero).
-// On return out[t * kTileRows + i] (shared, aliasing the pipeline) holds the
-// products for tokens t < kTokPad.
+struct TcShared {
+    uint64_t mma_done[8];  // per stage: the stage's MMAs have read it
+    uint32_t tmem;         // accumulator address
+    int fail;
+};
+
+// The tile's GEMM into tensor memory; rows_j[i] (shared) is the weight row of
+// tile row i (-1: zero). false if a bounded wait ran out (recorded).
 template <int MT>
-__device__ void gu_tile(const WideLaunch& L, const __nv_bfloat16* w, const int* rows_j, unsigned char* sm,
-                        float* out) {
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+__device__ bool gu_tile_tc(const WideLaunch& L, const __nv_bfloat16* w, const int* rows_j, unsigned char* sm,
+                           TcShared& ts) {
+    using C = TcCfg<MT>;
+    const int tid = threadIdx.x;
     const int d = L.d;
     const int nk = d / kTileK;
-    // this thread's copies per stage: 3 weight chunks, 2 activation chunks
-    const int wq = warp & 3, kh = warp >> 2;  // row tiles 3wq .. 3wq+2, K-steps 2kh, 2kh+1
-    const __nv_bfloat16* wsrc[3];
-    int wdst[3];
-    bool wok[3];
+    const __nv_bfloat16* wsrc[4];
+    int wdst[4];
+    bool wok[4];
 #pragma unroll
-    for (int i = 0; i < 3; ++i) {
-        const int q = tid + kGuThreads * i;  // 768 chunks: row q / 8, chunk q % 8
+    for (int i = 0; i < 4; ++i) {
+        const int q = tid + kGuThreads * i;  // 1024 chunks: row q / 8, chunk q % 8
         const int r = q >> 3, c = q & 7;
         const int j = rows_j[r];
         wok[i] = j >= 0;
         wsrc[i] = w + (size_t)(j >= 0 ? j : 0) * d + c * 8;
-        wdst[i] = GuSmem::kX + swz(r, c, 128);
+        wdst[i] = swz(r, c, 128);
     }
-    const __nv_bfloat16* xsrc[2];
-    int xdst[2];
-    bool xok[2];
+    constexpr int kXPer = (C::NP * 8 + kGuThreads - 1) / kGuThreads;
+    const __nv_bfloat16* xsrc[kXPer];
+    int xdst[kXPer];
+    bool xok[kXPer], xin[kXPer];
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
-        const int q = tid + kGuThreads * i;  // 512 chunks: token q / 8, chunk q % 8
+    for (int i = 0; i < kXPer; ++i) {
+        const int q = tid + kGuThreads * i;  // NP x 8 chunks: token q / 8, chunk q % 8
         const int t = q >> 3, c = q & 7;
+        xin[i] = t < C::NP;
         xok[i] = t < L.batch;
         xsrc[i] = L.x + (size_t)(t < L.batch ? t : 0) * d + c * 8;
-        xdst[i] = swz(t, c, 128);
+        xdst[i] = C::kA + swz(t, c, 128);
     }
     auto load = [&](int kst, int stage) {
-        unsigned char* base = sm + stage * GuSmem::kStage;
+        unsigned char* base = sm + stage * C::kStage;
         const int k0 = kst * kTileK;
 #pragma unroll
-        for (int i = 0; i < 3; ++i) cp16(base + wdst[i], wsrc[i] + k0, wok[i]);
+        for (int i = 0; i < 4; ++i) cp16(base + wdst[i], wsrc[i] + k0, wok[i]);
 #pragma unroll
-        for (int i = 0; i < 2; ++i) cp16(base + xdst[i], xsrc[i] + k0, xok[i]);
+        for (int i = 0; i < kXPer; ++i)
+            if (xin[i]) cp16(base + xdst[i], xsrc[i] + k0, xok[i]);
     };
-
-    float acc[MT][3][4];
-#pragma unroll
-    for (int a = 0; a < MT; ++a)
-#pragma unroll
-        for (int b = 0; b < 3; ++b)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) acc[a][b][e] = 0.0f;
-
-#pragma unroll
-    for (int s = 0; s < kStages - 1; ++s) {
+    const uint32_t sm0 = smem_addr(sm);
+    constexpr int S = C::kStages, D = kMmaLag;
+    bool ok = true;
+#pragma unroll 1
+    for (int s = 0; s < S - D; ++s) {
         if (s < nk) load(s, s);
         cp_commit();
     }
     for (int kst = 0; kst < nk; ++kst) {
-        cp_wait<kStages - 2>();
-        __syncthreads();  // the stage has landed for every thread; the oldest is free
-        if (kst + kStages - 1 < nk) load(kst + kStages - 1, (kst + kStages - 1) % kStages);
-        cp_commit();
-        const uint32_t xs = smem_addr(sm + (kst % kStages) * GuSmem::kStage);
-        const uint32_t ws = xs + GuSmem::kX;
-#pragma unroll
-        for (int k2 = 0; k2 < 2; ++k2) {
-            const int kk = 2 * kh + k2;
-            uint32_t af[MT][4];
-#pragma unroll
-            for (int mt = 0; mt < MT; ++mt) {
-                // a0..a3: tokens 0-7 / 8-15 of the m-tile at k chunk 2kk / 2kk+1
-                const int r = mt * 16 + (lane & 15);
-                ldsm4(xs + swz(r, 2 * kk + (lane >> 4), 128), af[mt]);
-            }
-            uint32_t bf[4], b2a, b2b;
-            {
-                // row tiles 3w, 3w+1: (rows, k lo), (rows, k hi) for each
-                const int r = wq * 24 + ((lane >> 4) << 3) + (lane & 7);
-                ldsm4(ws + swz(r, 2 * kk + ((lane >> 3) & 1), 128), bf);
-                const int r2 = wq * 24 + 16 + (lane & 7);
-                ldsm2(ws + swz(r2, 2 * kk + ((lane >> 3) & 1), 128), b2a, b2b);
-            }
-#pragma unroll
-            for (int mt = 0; mt < MT; ++mt) {
-                mma16816(acc[mt][0], af[mt], bf[0], bf[1]);
-                mma16816(acc[mt][1], af[mt], bf[2], bf[3]);
-                mma16816(acc[mt][2], af[mt], b2a, b2b);
-            }
-        }
-    }
-    cp_wait<0>();
-    __syncthreads();  // the pipeline buffers become the output tile
-    // the second K half first, then the first half adds its own (fixed order)
-    const int g = lane >> 2, t4 = lane & 3;
-    for (int half = 1; half >= 0; --half) {
-        if (kh == half) {
-#pragma unroll
-            for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-                for (int nt = 0; nt < 3; ++nt) {
-                    const int col = wq * 24 + nt * 8 + 2 * t4;
-                    const int tok = mt * 16 + g;
-                    float* o0 = out + tok * kTileRows + col;
-                    float* o1 = out + (tok + 8) * kTileRows + col;
-                    if (half == 1) {
-                        o0[0] = acc[mt][nt][0];
-                        o0[1] = acc[mt][nt][1];
-                        o1[0] = acc[mt][nt][2];
-                        o1[1] = acc[mt][nt][3];
-                    } else {
-                        o0[0] = acc[mt][nt][0] + o0[0];
-                        o0[1] = acc[mt][nt][1] + o0[1];
-                        o1[0] = acc[mt][nt][2] + o1[0];
-                        o1[1] = acc[mt][nt][3] + o1[1];
-                    }
-                }
-        }
+        cp_wait<S - D - 1>();      // k-block kst has landed (this thread's copies)
+        fence_proxy_async_smem();  // ... and is visible to the tensor cores
         __syncthreads();
+        if (ts.fail) {             // a bounded wait ran out somewhere (set before the barrier)
+            ok = false;
+            break;
+        }
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t a0 = sm0 + (kst % S) * C::kStage;
+            const uint64_t ad = sdesc_k128(a0), bd = sdesc_k128(a0 + C::kA);
+#pragma unroll
+            for (int kk = 0; kk < kTileK / 16; ++kk)  // 32 bytes of each row per MMA
+                tc_mma(ts.tmem, ad + 2 * kk, bd + 2 * kk, C::kIdesc, (kst | kk) != 0);
+            tc_commit(&ts.mma_done[kst % S]);
+        }
+        // refill the stage of k-block kst - D, whose MMAs were issued D
+        // iterations ago, so the wait rarely stalls on the MMA pipeline
+        const int nxt = kst + S - D;
+        if (nxt < nk) {
+            if (kst >= D && !mbar_wait(&ts.mma_done[(kst - D) % S], (unsigned)((kst - D) / S) & 1u)) ts.fail = 1;
+            load(nxt, nxt % S);
+        }
+        cp_commit();
     }
+    // every MMA done (the last commit covers all earlier ones)
+    if (ok && !mbar_wait(&ts.mma_done[(nk - 1) % S], (unsigned)((nk - 1) / S) & 1u)) ts.fail = 1;
+    cp_wait<0>();
+    __syncthreads();
+    ok = ok && ts.fail == 0;
+    if (!ok && tid == 0) atomicOr(L.status, kStatusTimeout);
+    tc_fence_after();
+    return ok;
+}
+
+// tensor memory and barriers for the tile; warp 0 allocates
+template <int MT>
+__device__ void tc_setup(TcShared& ts) {
+    if (threadIdx.x < kWarp) {
+        tc_alloc(&ts.tmem, TcCfg<MT>::kCols);
+        tc_relinquish();
+    }
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < TcCfg<MT>::kStages; ++s) mbar_init(&ts.mma_done[s], 1);
+        ts.fail = 0;
+        mbar_fence_init();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+}
+template <int MT>
+__device__ void tc_teardown(TcShared& ts) {
+    tc_fence_before();
+    __syncthreads();
+    if (threadIdx.x < kWarp) {
+        tc_fence_after();
+        tc_dealloc(ts.tmem, TcCfg<MT>::kCols);
+    }
+}
+
+__device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
+    const uint32_t a = smem_addr(p);
+    return p + ((1024u - (a & 1023u)) & 1023u);
 }
 
 template <int MT>
 __global__ void __launch_bounds__(kGuThreads) k_wide_gate(const WideLaunch L) {
-    extern __shared__ __align__(128) unsigned char sm[];
-    __shared__ int rows_j[kTileRows];
+    extern __shared__ __align__(1024) unsigned char sm_raw[];
+    __shared__ int rows_j[kTcRows];
+    __shared__ unsigned s_union[kTcRows / 32];
+    __shared__ TcShared ts;
+    unsigned char* sm = align1024(sm_raw);
     pdl_wait();
     pdl_launch_dependents();
-    const int p0 = blockIdx.x * kTileRows;
-    const int tid = threadIdx.x;
-    if (tid < kTileRows) rows_j[tid] = p0 + tid < L.n_rows ? row_of(L, p0 + tid) : -1;
-    __syncthreads();
-    float* out = reinterpret_cast<float*>(sm);
-    gu_tile<MT>(L, L.wg, rows_j, sm, out);
-    // g values, per-token gate bitmap bytes (and cleared both bytes) for the tile
-    const int n_in = min(kTileRows, L.n_rows - p0);
-    for (int q = tid; q < L.batch * kTileRows; q += kGuThreads) {
-        const int t = q / kTileRows, i = q % kTileRows;
-        if (i < n_in) L.gval[(size_t)t * L.n_rows + p0 + i] = out[t * kTileRows + i];
-    }
-    const int n_bytes = (n_in + 7) / 8;
-    for (int q = tid; q < L.batch * n_bytes; q += kGuThreads) {
-        const int t = q / n_bytes, b = q % n_bytes;
-        unsigned bits = 0u;
-        for (int r = 0; r < 8; ++r) {
-            const int i = b * 8 + r;
-            if (i < n_in && rows_j[i] >= 0 && out[t * kTileRows + i] > 0.0f) bits |= 1u << r;
-        }
-        L.gbits[(size_t)t * L.nbytes + p0 / 8 + b] = (uint8_t)bits;
-        L.bbits[(size_t)t * L.nbytes + p0 / 8 + b] = 0;
-    }
-    for (int b = tid; b < n_bytes; b += kGuThreads) {
-        unsigned u = 0u;
-        for (int t = 0; t < L.batch; ++t)
-            for (int r = 0; r < 8; ++r) {
-                const int i = b * 8 + r;
-                if (i < n_in && rows_j[i] >= 0 && out[t * kTileRows + i] > 0.0f) u |= 1u << r;
+    const int p0 = blockIdx.x * kTcRows;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (tid < kTcRows) rows_j[tid] = p0 + tid < L.n_rows ? row_of(L, p0 + tid) : -1;
+    if (tid < kTcRows / 32) s_union[tid] = 0u;
+    tc_setup<MT>(ts);
+    const bool ok = gu_tile_tc<MT>(L, L.wg, rows_j, sm, ts);
+    // warp w reads tile rows 32 (w % 4) .. + 31, token tiles w / 4, w / 4 + 2
+    const int q = warp & 3, i = 32 * q + lane, p = p0 + i;
+    const int n_in = min(kTcRows, L.n_rows - p0);
+    const bool row_in = i < n_in && rows_j[i] >= 0;
+    unsigned uw = 0u;
+    const int word = (p0 + 32 * q) / 32;  // bitmap word of rows p0 + 32 q .. + 31
+    const bool word_in = p0 + 32 * q < L.n_rows;
+    if (ok) {
+        for (int mt = warp >> 2; mt < MT; mt += 2) {
+            float v[16];
+            tc_ld16(ts.tmem + ((uint32_t)(32 * q) << 16) + 16 * mt, v);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int t = 16 * mt + e;
+                if (t < L.batch && i < n_in) L.gval[(size_t)t * L.n_rows + p] = v[e];
+                const unsigned bits = __ballot_sync(0xffffffffu, t < L.batch && row_in && v[e] > 0.0f);
+                if (t < L.batch && lane == 0 && word_in) {
+                    reinterpret_cast<unsigned*>(L.gbits + (size_t)t * L.nbytes)[word] = bits;
+                    reinterpret_cast<unsigned*>(L.bbits + (size_t)t * L.nbytes)[word] = 0u;
+                }
+                uw |= bits;
             }
-        L.ugbits[p0 / 8 + b] = (uint8_t)u;
-        L.ubits[p0 / 8 + b] = 0;
+        }
+        if (lane == 0 && uw) atomicOr(&s_union[q], uw);
     }
+    __syncthreads();
+    if (ok && warp < 4 && lane == 0 && word_in) {
+        reinterpret_cast<unsigned*>(L.ugbits)[word] = s_union[q];
+        reinterpret_cast<unsigned*>(L.ubits)[word] = 0u;
+    }
+    tc_teardown<MT>(ts);
 }
 
 template <int MT>
 __global__ void __launch_bounds__(kGuThreads) k_wide_up(const WideLaunch L) {
-    extern __shared__ __align__(128) unsigned char sm[];
-    __shared__ int rows_j[kTileRows];
-    __shared__ int pos[kTileRows];
+    extern __shared__ __align__(1024) unsigned char sm_raw[];
+    __shared__ int rows_j[kTcRows];
+    __shared__ int pos[kTcRows];
     __shared__ int s_part[kGuThreads + 1];
+    __shared__ TcShared ts;
+    unsigned char* sm = align1024(sm_raw);
     pdl_wait();
     pdl_launch_dependents();
-    const int tid = threadIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const unsigned* ug = reinterpret_cast<const unsigned*>(L.ugbits);
     const BitScan bs = bit_scan<kGuThreads>(ug, L.n_rows, s_part);
-    const int i0 = blockIdx.x * kTileRows;
+    const int i0 = blockIdx.x * kTcRows;
     if (i0 >= bs.total) return;  // the union gate-active list is shorter
-    const int n_in = min(kTileRows, bs.total - i0);
-    if (tid < kTileRows) pos[tid] = -1;
+    const int n_in = min(kTcRows, bs.total - i0);
+    if (tid < kTcRows) pos[tid] = -1;
     __syncthreads();
     bit_emit(ug, L.n_rows, bs, i0, i0 + n_in, pos);
     __syncthreads();
-    if (tid < kTileRows) rows_j[tid] = pos[tid] >= 0 ? (L.rows ? L.rows[pos[tid]] : pos[tid]) : -1;
-    __syncthreads();
-    float* out = reinterpret_cast<float*>(sm);
-    gu_tile<MT>(L, L.wu, rows_j, sm, out);
+    if (tid < kTcRows) rows_j[tid] = pos[tid] >= 0 ? (L.rows ? L.rows[pos[tid]] : pos[tid]) : -1;
+    tc_setup<MT>(ts);
+    const bool ok = gu_tile_tc<MT>(L, L.wu, rows_j, sm, ts);
     // c = g u where both are positive (Eq. 2), split into bf16 hi + lo
+    const int q = warp & 3, i = 32 * q + lane;
+    const int p = pos[i];
     unsigned* bb = reinterpret_cast<unsigned*>(L.bbits);
     unsigned* ub = reinterpret_cast<unsigned*>(L.ubits);
-    for (int q = tid; q < n_in * kTokPad; q += kGuThreads) {
-        const int i = q / kTokPad, t = q % kTokPad;
-        const int p = pos[i];
-        float c = 0.0f;
-        if (t < L.batch) {
-            const float gv = L.gval[(size_t)t * L.n_rows + p];
-            const float uv = out[t * kTileRows + i];
-            if (gv > 0.0f && uv > 0.0f) {
-                c = gv * uv;
-                atomicOr(bb + (size_t)t * (L.nbytes / 4) + p / 32, 1u << (p % 32));
-                atomicOr(ub + p / 32, 1u << (p % 32));
+    if (ok) {
+        for (int mt = warp >> 2; mt < kTokPad / 16; mt += 2) {
+            float v[16];
+            if (mt < MT) tc_ld16(ts.tmem + ((uint32_t)(32 * q) << 16) + 16 * mt, v);
+            if (p < 0) continue;
+            __align__(16) __nv_bfloat16 hi[16], lo[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int t = 16 * mt + e;
+                float c = 0.0f;
+                if (mt < MT && t < L.batch) {
+                    const float gv = L.gval[(size_t)t * L.n_rows + p];
+                    const float uv = v[e];
+                    if (gv > 0.0f && uv > 0.0f) {
+                        c = gv * uv;
+                        atomicOr(bb + (size_t)t * (L.nbytes / 4) + p / 32, 1u << (p % 32));
+                        atomicOr(ub + p / 32, 1u << (p % 32));
+                    }
+                }
+                hi[e] = __float2bfloat16_rn(c);
+                lo[e] = __float2bfloat16_rn(c - __bfloat162float(hi[e]));
             }
+            uint4* dh = reinterpret_cast<uint4*>(L.c_hi + (size_t)p * kTokPad + 16 * mt);
+            uint4* dl = reinterpret_cast<uint4*>(L.c_lo + (size_t)p * kTokPad + 16 * mt);
+            dh[0] = reinterpret_cast<const uint4*>(hi)[0];
+            dh[1] = reinterpret_cast<const uint4*>(hi)[1];
+            dl[0] = reinterpret_cast<const uint4*>(lo)[0];
+            dl[1] = reinterpret_cast<const uint4*>(lo)[1];
         }
-        const __nv_bfloat16 hi = __float2bfloat16_rn(c);
-        L.c_hi[(size_t)p * kTokPad + t] = hi;
-        L.c_lo[(size_t)p * kTokPad + t] = __float2bfloat16_rn(c - __bfloat162float(hi));
     }
+    tc_teardown<MT>(ts);
 }
 
 // ---------------------------------------------------------------------------
@@ -568,9 +667,9 @@ cudaError_t launch(K kernel, int grid, int threads, size_t smem, cudaStream_t st
 
 template <int MT>
 cudaError_t run_t(const WideLaunch& L, cudaStream_t stream, bool pdl) {
-    const int gu_grid = (L.n_rows + kTileRows - 1) / kTileRows;
-    cudaError_t e = launch(k_wide_gate<MT>, gu_grid, kGuThreads, GuSmem::kBytes, stream, pdl, L);
-    if (e == cudaSuccess) e = launch(k_wide_up<MT>, gu_grid, kGuThreads, GuSmem::kBytes, stream, true, L);
+    const int gu_grid = (L.n_rows + kTcRows - 1) / kTcRows;
+    cudaError_t e = launch(k_wide_gate<MT>, gu_grid, kGuThreads, TcCfg<MT>::kBytes, stream, pdl, L);
+    if (e == cudaSuccess) e = launch(k_wide_up<MT>, gu_grid, kGuThreads, TcCfg<MT>::kBytes, stream, true, L);
     if (e == cudaSuccess)
         e = launch(k_wide_down<MT>, (L.d / kDownCols) * L.ks, kDownThreads, DnSmem::kBytes, stream, true, L);
     if (e == cudaSuccess) {
@@ -582,8 +681,8 @@ cudaError_t run_t(const WideLaunch& L, cudaStream_t stream, bool pdl) {
 
 template <int MT>
 cudaError_t prepare_t() {
-    cudaError_t e = cudaFuncSetAttribute(k_wide_gate<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, GuSmem::kBytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_wide_up<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, GuSmem::kBytes);
+    cudaError_t e = cudaFuncSetAttribute(k_wide_gate<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<MT>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_wide_up<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<MT>::kBytes);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_wide_down<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, DnSmem::kBytes);
     return e;
 }

@@ -78,6 +78,7 @@ def test_argument_validation_without_device(lib):
     assert lib.ts_moe_get_error(None, None) == TS_ERR_INVALID_ARG
     assert lib.ts_graph_launch(None, None) == TS_ERR_INVALID_ARG
     assert lib.ts_graph_capture_stack(None, None, 0, None, 0, None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_graph_capture_stack_fused(None, None, 0, None, 0, None, None) == TS_ERR_INVALID_ARG
     lib.ts_ffn_destroy(None)
     lib.ts_moe_destroy(None)
     lib.ts_graph_destroy(None)
