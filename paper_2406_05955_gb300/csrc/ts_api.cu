@@ -406,7 +406,7 @@ ts_status read_status(unsigned* status_dev, cudaStream_t stream) {
 // rows (all, or the list). `next` is the following layer when it runs dense
 // (its first W_gate rows are then prefetched into L2), else nullptr.
 ts_status stack_layer(ts_ffn* h, const ts_ffn* next, float* hres, int batch, const int32_t* rows, int nr,
-                      cudaStream_t stream, bool rows_ready) {
+                      cudaStream_t stream, bool rows_ready, bool h_ready = false) {
     if (use_wide(h, batch)) {
         WideLaunch L = wide_launch(h, batch, rows, nr);
         L.x = h->w_x;
@@ -423,6 +423,7 @@ ts_status stack_layer(ts_ffn* h, const ts_ffn* next, float* hres, int batch, con
     a.norm_from_h = 1;
     a.residual_out = 1;
     a.rows_ready = rows != nullptr && rows_ready ? 1 : 0;
+    a.h_ready = h_ready ? 1 : 0;
     if (next != nullptr && batch <= kMaxPass && h->dt != TS_INT4) {
         a.next_wg = next->wg;
         a.next_n_rows = next->m;
@@ -893,7 +894,8 @@ ts_status ts_stack_forward_predicted(ts_ffn* const* layers, ts_predictor* const*
         PredictLaunch q = predict_launch(preds[l], batch, K[l], lists[l], nullptr);
         q.h = hres;
         ts_status st = cuda_status(launch_predict(q, elem_size(preds[l]->dt), stream, true));
-        if (st == TS_OK) st = stack_layer(h, nullptr, hres, batch, lists[l], K[l], stream, false);
+        // the predictor's three kernels ran after the last writer of h
+        if (st == TS_OK) st = stack_layer(h, nullptr, hres, batch, lists[l], K[l], stream, false, true);
         if (st != TS_OK) return st;
     }
     return TS_OK;

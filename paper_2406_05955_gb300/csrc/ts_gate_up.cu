@@ -1696,7 +1696,11 @@ __device__ void consume_rows(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned 
     }
 }
 
-template <typename T, int NT>
+// PRE: the launch is the predicted stack's (a list made by the kernel just
+// before, over a residual that was final before it): the activations are
+// staged first and only then is the list waited for. A separate
+// instantiation, so that the other launches keep their register budget.
+template <typename T, int NT, bool PRE = false>
 __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(const FfnLaunch a, const RowsCfg rc) {
     constexpr int C = GateUpWarps<NT>::C;
     __shared__ GateUpShared<NT> sh;
@@ -1716,7 +1720,8 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(co
         mbar_fence_init();
     }
     const bool early = (a.rows == nullptr || a.rows_ready) && a.route == nullptr;
-    if (!early) pdl_wait();
+    constexpr bool pre_stage = PRE;
+    if (!early && !pre_stage) pdl_wait();
     resolve_experts(a, sh.es);
     pdl_launch_dependents();
 
@@ -1729,10 +1734,22 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(co
     const int ctid = threadIdx.x - kWarp;
     const int cthreads = C * kWarp;
     const int x_tok0 = a.route ? 0 : a.tok0;
+    if (pre_stage) {
+        for (int t = 0; t < n_x; ++t) {
+            float* xrow = xs + (size_t)t * rc.xs_stride;
+            stage_act_row<T>(a.h + (size_t)(x_tok0 + t) * a.d, nullptr, a.d, ctid, cthreads, sh.red,
+                             [&](int i, float v) { xrow[xs_index<T>(i)] = v; });
+        }
+        named_bar_sync(1, cthreads);
+        pdl_wait();
+    }
     // Stage the activations; first_rows() (the first weight-row copies) runs
     // once, right after the first activation loads are issued.
     auto stage = [&](auto&& first_rows) {
-        if (early) pdl_wait();
+        if (pre_stage) {  // staged already
+            first_rows();
+            return;
+        }
         bool started = false;
         auto once = [&]() {
             if (!started) {
@@ -1740,6 +1757,7 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(co
                 first_rows();
             }
         };
+        if (early) pdl_wait();
         for (int t = 0; t < n_x; ++t) {
             float* xrow = xs + (size_t)t * rc.xs_stride;
             stage_act_row<T>(a.norm_from_h ? a.h + (size_t)(x_tok0 + t) * a.d : nullptr,
@@ -2065,7 +2083,9 @@ static cudaError_t launch_rows_t(const FfnLaunch& a, int grid, cudaStream_t stre
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = attr;
     lc.numAttrs = pdl ? 1 : 0;
-    return cudaLaunchKernelEx(&lc, k_gate_up_rows<T, NT>, a, rc);
+    if (a.h_ready && a.norm_from_h && a.route == nullptr && a.rows != nullptr && !a.rows_ready)
+        return cudaLaunchKernelEx(&lc, k_gate_up_rows<T, NT, true>, a, rc);
+    return cudaLaunchKernelEx(&lc, k_gate_up_rows<T, NT, false>, a, rc);
 }
 
 template <int NT>
@@ -2158,8 +2178,10 @@ cudaError_t prepare_gate_up(int optin_smem) {
     const int dyn = optin_smem - kSmemMargin;
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_rows<__nv_bfloat16, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_rows<__nv_bfloat16, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_rows<__nv_bfloat16, 1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_rows<__nv_bfloat16, 2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_rows<__nv_bfloat16, 1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_rows<__nv_bfloat16, 2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_stack_rows<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_stack_rows<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gate_up_q4w<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);

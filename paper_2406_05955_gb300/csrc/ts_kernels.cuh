@@ -90,6 +90,11 @@ struct FfnLaunch {
     // before waiting for them (stack layers after the first, with the
     // caller's lists).
     int rows_ready;
+    // Nonzero when the residual h (stack mode) was final before the kernels
+    // preceding this launch in the stream ran (the predicted stack: the
+    // predictor's kernels sit between the last writer of h and this launch),
+    // so the activations may be staged before waiting for them.
+    int h_ready;
     // Stack mode: the next layer's W_gate (nullptr: none), its row count and
     // its gate+up grid. The gathered down kernel (passes of 4-8 tokens),
     // before waiting for the gate+up kernel, prefetches into L2 the first

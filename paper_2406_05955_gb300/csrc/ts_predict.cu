@@ -12,6 +12,8 @@
 //                  key bits (HBM-bound: reads W2 once)
 //   k_pred_select  one CTA: MSB-first 8-bit radix select of the K-th largest
 //                  key, then an ordered emission of the selected ids
+//                  (k_pred_select_hist, led by the score kernel's histogram,
+//                  when m <= 16384)
 #include <math.h>
 
 #include <algorithm>
@@ -145,6 +147,7 @@ __global__ void __launch_bounds__(kPredThreads) k_pred_score(const PredictLaunch
     extern __shared__ __align__(16) float hs[];  // [NB][r]
     constexpr int N = Vec<T>::N;
     constexpr int RG = STEPS >= 8 ? 1 : 8 / STEPS;
+    constexpr int WARPS = kPredWarps;
     const int r = p.r, m = p.m;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int groups = (m + RG - 1) / RG;
@@ -161,7 +164,7 @@ __global__ void __launch_bounds__(kPredThreads) k_pred_score(const PredictLaunch
     };
     // W2 does not depend on earlier kernels: this warp's first group of rows
     // is loaded before the wait, while the hidden-layer kernel runs.
-    int g = blockIdx.x * kPredWarps + warp;
+    int g = blockIdx.x * WARPS + warp;
     if (g < groups) load(g);
     pdl_launch_dependents();
     pdl_wait();
@@ -177,7 +180,7 @@ __global__ void __launch_bounds__(kPredThreads) k_pred_score(const PredictLaunch
     __syncthreads();
 
     bool loaded = true;
-    for (; g < groups; g += gridDim.x * kPredWarps) {
+    for (; g < groups; g += gridDim.x * WARPS) {
         const int j0 = g * RG;
         if (!loaded) load(g);
         loaded = false;
@@ -384,20 +387,20 @@ __device__ __forceinline__ void block_scan2(int a, int b, int& ea, int& eb, int&
 //      number of keys above it.
 //   2. The keys in bin B (usually a few hundred) are compacted into shared
 //      memory, and the (K - above)-th largest of their low 20 bits is found
-//      bit by bit from the top (keep bit b if enough candidates are >= the
-//      prefix with b set), which gives the K-th largest key T.
+//      digit by digit from the top (8, 8, then 4 bits: a shared histogram of
+//      the next digit among the candidates matching the digits so far),
+//      which gives the K-th largest key T.
 //   3. A block scan of the per-thread counts of keys > T and == T places
 //      every kept id in ascending order.
 // Absent ids hold key 0 and are never counted.
 constexpr int kSelKeys = 16;
 
-__global__ void __launch_bounds__(kSelThreads) k_pred_select_hist(const PredictLaunch p) {
-    extern __shared__ unsigned cand[];  // [m] low 20 bits of the keys in bin B
+// kSelThreads threads; cand: [m] unsigned of shared memory. Keys and the
+// histogram are read at L2 (other CTAs may have just written them).
+__device__ void select_hist_body(const PredictLaunch& p, unsigned* cand) {
     __shared__ int s_a[kSelWarps], s_b[kSelWarps], s_tot[2];
-    __shared__ int s_cnt[2][kSelWarps];
+    __shared__ unsigned s_dig[256], s_sel[2];
     __shared__ int s_bin, s_above;
-    pdl_wait();
-    pdl_launch_dependents();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int m = p.m, K = p.K;
     const unsigned full = 0xffffffffu;
@@ -405,7 +408,7 @@ __global__ void __launch_bounds__(kSelThreads) k_pred_select_hist(const PredictL
     const int i0 = tid * per;
     unsigned key[kSelKeys];
 #pragma unroll
-    for (int q = 0; q < kSelKeys; ++q) key[q] = (q < per && i0 + q < m) ? p.key[i0 + q] : 0u;
+    for (int q = 0; q < kSelKeys; ++q) key[q] = (q < per && i0 + q < m) ? __ldcg(p.key + i0 + q) : 0u;
     constexpr int BPT = kPredHistBins / kSelThreads;  // bins per thread
     int hv[BPT], hsum = 0;
 #pragma unroll
@@ -413,7 +416,7 @@ __global__ void __launch_bounds__(kSelThreads) k_pred_select_hist(const PredictL
         hv[q] = 0;
 #pragma unroll
         for (int part = 0; part < kPredHistParts; ++part)
-            hv[q] += (int)p.hist[part * kPredHistBins + kPredHistBins - 1 - (BPT * tid + q)];
+            hv[q] += (int)__ldcg(p.hist + part * kPredHistBins + kPredHistBins - 1 - (BPT * tid + q));
         hsum += hv[q];
     }
     int above, unused, htot, unused2;
@@ -440,17 +443,52 @@ __global__ void __launch_bounds__(kSelThreads) k_pred_select_hist(const PredictL
         if (key[q] != 0u && (key[q] >> 20) == B) cand[off++] = key[q] & 0xfffffu;
     __syncthreads();
 
-    unsigned L = 0u;
-    for (int b = 19; b >= 0; --b) {
-        const unsigned cv = L | (1u << b);
-        int cnt = 0;
-        for (int i = tid; i < n_c; i += kSelThreads) cnt += cand[i] >= cv ? 1 : 0;
-        cnt = (int)__reduce_add_sync(full, (unsigned)cnt);
-        // two buffers: a step's writes cannot meet the previous step's reads
-        if (lane == 0) s_cnt[b & 1][warp] = cnt;
+    // the need_in_bin-th largest of the candidates' low 20 bits, by digits of
+    // 8, 8 and 4 bits from the top: count the candidates that match the
+    // digits found so far into a histogram of the next digit, then take the
+    // digit holding the remaining rank (counting from the top)
+    unsigned L = 0u, Lmask = 0u;
+    int rem = need_in_bin;
+    for (int pass = 0; pass < 3; ++pass) {
+        const int shift = pass == 0 ? 12 : (pass == 1 ? 4 : 0);
+        const int nb = pass == 2 ? 16 : 256;
+        for (int i = tid; i < 256; i += kSelThreads) s_dig[i] = 0u;
         __syncthreads();
-        const int tot = (int)__reduce_add_sync(full, (unsigned)s_cnt[b & 1][lane]);
-        if (tot >= need_in_bin) L = cv;
+        for (int i = tid; i < n_c; i += kSelThreads) {
+            const unsigned cv = cand[i];
+            if ((cv & Lmask) == L) atomicAdd(&s_dig[(cv >> shift) & (unsigned)(nb - 1)], 1u);
+        }
+        __syncthreads();
+        if (warp == 0) {
+            // lane l holds the counts of digits nb-1-8l .. nb-8-8l (highest first)
+            unsigned c8[8], sum = 0u;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int dgt = nb - 1 - 8 * lane - q;
+                c8[q] = dgt >= 0 ? s_dig[dgt] : 0u;
+                sum += c8[q];
+            }
+            unsigned incl = sum;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const unsigned nv = __shfl_up_sync(full, incl, o);
+                if (lane >= o) incl += nv;
+            }
+            unsigned above_l = incl - sum;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                if (above_l < (unsigned)rem && (unsigned)rem <= above_l + c8[q]) {
+                    s_sel[0] = (unsigned)(nb - 1 - 8 * lane - q);
+                    s_sel[1] = (unsigned)rem - above_l;
+                }
+                above_l += c8[q];
+            }
+        }
+        __syncthreads();
+        L |= s_sel[0] << shift;
+        Lmask |= (unsigned)(nb - 1) << shift;
+        rem = (int)s_sel[1];
+        __syncthreads();  // s_dig and s_sel are rewritten by the next pass
     }
     const unsigned T = (B << 20) | L;
 
@@ -475,6 +513,13 @@ __global__ void __launch_bounds__(kSelThreads) k_pred_select_hist(const PredictL
             ++run_eq;
         }
     }
+}
+
+__global__ void __launch_bounds__(kSelThreads) k_pred_select_hist(const PredictLaunch p) {
+    extern __shared__ unsigned cand[];  // [m] low 20 bits of the keys in bin B
+    pdl_wait();
+    pdl_launch_dependents();
+    select_hist_body(p, cand);
 }
 
 template <typename T, int NB>
@@ -522,14 +567,11 @@ cudaError_t prepare_nb(int optin_smem) {
     cudaError_t e = cudaFuncSetAttribute(k_pred_hidden<T, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          optin_smem - kSmemSlack);
     const int score_smem = NB * 8 * kWarp * Vec<T>::N * (int)sizeof(float);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_pred_score<T, NB, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, score_smem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_pred_score<T, NB, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, score_smem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_pred_score<T, NB, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, score_smem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_pred_score<T, NB, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, score_smem);
+    const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_pred_score<T, NB, 1>, a, score_smem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_pred_score<T, NB, 2>, a, score_smem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_pred_score<T, NB, 4>, a, score_smem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_pred_score<T, NB, 8>, a, score_smem);
     return e;
 }
 

@@ -172,6 +172,9 @@ __device__ void bit_emit(const unsigned* words, int n_bits, const BitScan& b, in
 constexpr int kTcRows = 128;  // weight rows per tile: the MMA's M
 constexpr int kMmaLag = 2;    // a stage is refilled kMmaLag k-blocks after its MMAs were issued
 
+constexpr int kTcStages = 8;  // most pipeline stages of a tensor-core tile
+constexpr int kTcSmem = 192 * 1024;  // pipeline bytes of a tensor-core tile
+
 __device__ __forceinline__ void tc_alloc(uint32_t* dst, uint32_t ncols) {  // warp-wide
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(dst)), "r"(ncols)
                  : "memory");
@@ -232,7 +235,7 @@ struct TcCfg {
     static constexpr int kA = kTcRows * 128;           // 16 KB of weight rows per stage
     static constexpr int kB = NP * 128;                // activations per stage
     static constexpr int kStage = kA + kB;
-    static constexpr int kStages = (192 * 1024) / kStage > 8 ? 8 : (192 * 1024) / kStage;
+    static constexpr int kStages = kTcSmem / kStage > kTcStages ? kTcStages : kTcSmem / kStage;
     static constexpr int kBytes = kStages * kStage + 1024;  // + slack to align the tiles to 1024 bytes
     static constexpr uint32_t kCols = NP <= 16 ? 32 : (NP <= 32 ? 64 : 128);  // tensor-memory columns: a power of 2, >= 2 N
     static constexpr uint32_t kIdesc = idesc_bf16_f32(kTcRows, NP);
@@ -440,6 +443,49 @@ __global__ void __launch_bounds__(kGuThreads) k_wide_up(const WideLaunch L) {
     unsigned* bb = reinterpret_cast<unsigned*>(L.bbits);
     unsigned* ub = reinterpret_cast<unsigned*>(L.ubits);
     if (ok) {
+      // A warp whose 32 rows fill one bitmap word (the list is dense there:
+      // nearly every neuron gate-active) ORs its bits together, so the word
+      // takes one atomic per token instead of 32 contending ones; elsewhere
+      // one atomic per both-active (row, token) measured faster.
+      const int w32 = p >= 0 ? p / 32 : -1;
+      const unsigned same = __match_any_sync(0xffffffffu, w32);
+      if (same == 0xffffffffu && w32 >= 0) {
+        const unsigned bit = 1u << (p % 32);
+        const bool leader = (__ffs(same) - 1) == lane;
+        unsigned any_both = 0u;
+        for (int mt = warp >> 2; mt < kTokPad / 16; mt += 2) {
+            float v[16];
+            if (mt < MT) tc_ld16(ts.tmem + ((uint32_t)(32 * q) << 16) + 16 * mt, v);
+            __align__(16) __nv_bfloat16 hi[16], lo[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int t = 16 * mt + e;
+                float c = 0.0f;
+                if (p >= 0 && mt < MT && t < L.batch) {
+                    const float gv = L.gval[(size_t)t * L.n_rows + p];
+                    const float uv = v[e];
+                    if (gv > 0.0f && uv > 0.0f) c = gv * uv;
+                }
+                const unsigned mine = c > 0.0f ? bit : 0u;
+                any_both |= mine;
+                if (mt < MT && t < L.batch) {
+                    const unsigned word_bits = __reduce_or_sync(same, mine);
+                    if (leader && word_bits) atomicOr(bb + (size_t)t * (L.nbytes / 4) + w32, word_bits);
+                }
+                hi[e] = __float2bfloat16_rn(c);
+                lo[e] = __float2bfloat16_rn(c - __bfloat162float(hi[e]));
+            }
+            if (p < 0) continue;
+            uint4* dh = reinterpret_cast<uint4*>(L.c_hi + (size_t)p * kTokPad + 16 * mt);
+            uint4* dl = reinterpret_cast<uint4*>(L.c_lo + (size_t)p * kTokPad + 16 * mt);
+            dh[0] = reinterpret_cast<const uint4*>(hi)[0];
+            dh[1] = reinterpret_cast<const uint4*>(hi)[1];
+            dl[0] = reinterpret_cast<const uint4*>(lo)[0];
+            dl[1] = reinterpret_cast<const uint4*>(lo)[1];
+        }
+        const unsigned union_bits = __reduce_or_sync(same, any_both);
+        if (leader && union_bits) atomicOr(ub + w32, union_bits);
+      } else {
         for (int mt = warp >> 2; mt < kTokPad / 16; mt += 2) {
             float v[16];
             if (mt < MT) tc_ld16(ts.tmem + ((uint32_t)(32 * q) << 16) + 16 * mt, v);
@@ -468,6 +514,7 @@ __global__ void __launch_bounds__(kGuThreads) k_wide_up(const WideLaunch L) {
             dl[0] = reinterpret_cast<const uint4*>(lo)[0];
             dl[1] = reinterpret_cast<const uint4*>(lo)[1];
         }
+      }
     }
     tc_teardown<MT>(ts);
 }
@@ -615,6 +662,174 @@ __global__ void __launch_bounds__(kDownThreads) k_wide_down(const WideLaunch L) 
         }
 }
 
+// ---------------------------------------------------------------------------
+// down on the 5th-generation tensor cores: D[n][t] = sum over the slice's
+// union both-active rows p of W_down[row p][n0 + n] c_t,p, for 128 output
+// columns (the MMA's M) and all tokens (N), both operands MN-major: a K-row
+// of the A tile is 256 contiguous bytes of a W_down row, a K-row of the B
+// tile the 128 bytes of c (64 tokens) of that row. c enters twice, as its
+// bf16 hi and lo parts, into the same accumulator.
+// Stage (64 list rows): A as two 64-column halves of 64 rows x 128 bytes
+// (128-byte swizzle, 8-row atoms), then the c hi and lo tiles (64 rows x
+// 128 bytes each).
+// ---------------------------------------------------------------------------
+constexpr int kTcDownCols = 128;  // output columns per CTA: the MMA's M
+constexpr int kTcDownK = 64;      // list rows per stage
+constexpr int kTcDownPiece = 2048;  // list entries resolved at a time
+
+template <int MT>
+struct TcDownCfg {
+    static constexpr int NP = 16 * MT;
+    static constexpr int kAHalf = kTcDownK * 128;  // 8 KB: 64 rows x 64 columns
+    static constexpr int kA = 2 * kAHalf;
+    static constexpr int kC = kTcDownK * 128;      // 8 KB: 64 rows x 64 tokens
+    static constexpr int kStage = kA + 2 * kC;     // 32 KB
+    static constexpr int kStages = kTcSmem / kStage > kTcStages ? kTcStages : kTcSmem / kStage;
+    static constexpr int kBytes = kStages * kStage + 1024;
+    static constexpr uint32_t kCols = NP <= 16 ? 32 : (NP <= 32 ? 64 : 128);
+    // bf16 A and B, both MN-major (bits 15, 16), fp32 D, M = 128, N = NP
+    static constexpr uint32_t kIdesc = idesc_bf16_f32(kTcDownCols, NP) | (1u << 15) | (1u << 16);
+};
+
+// MN-major tile with the 128-byte swizzle: 64 contiguous MN elements per
+// 128-byte K-row, 8 K-rows per 1024-byte atom; `lbo` bytes between 64-element
+// MN blocks, 1024 bytes between 8-row K groups
+__device__ __forceinline__ uint64_t sdesc_mn128(uint32_t saddr, uint32_t lbo) {
+    uint64_t dsc = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    dsc |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+    dsc |= (uint64_t)(1024 >> 4) << 32;
+    dsc |= (uint64_t)1 << 46;
+    dsc |= (uint64_t)2 << 61;
+    return dsc;
+}
+
+template <int MT>
+__global__ void __launch_bounds__(kGuThreads) k_wide_down_tc(const WideLaunch L) {
+    using C = TcDownCfg<MT>;
+    extern __shared__ __align__(1024) unsigned char sm_raw[];
+    __shared__ int pos[kTcDownPiece];
+    __shared__ int s_part[kGuThreads + 1];
+    __shared__ TcShared ts;
+    unsigned char* sm = align1024(sm_raw);
+    pdl_wait();
+    pdl_launch_dependents();
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int d = L.d;
+    const int n_tiles = d / kTcDownCols;
+    const int n0 = (blockIdx.x % n_tiles) * kTcDownCols;
+    const int sl = blockIdx.x / n_tiles;
+    const unsigned* ub = reinterpret_cast<const unsigned*>(L.ubits);
+    const BitScan bs = bit_scan<kGuThreads>(ub, L.n_rows, s_part);
+    const int k_begin = (int)((long long)bs.total * sl / L.ks);
+    const int k_end = (int)((long long)bs.total * (sl + 1) / L.ks);
+    const int n_list = k_end - k_begin;
+    const int nk = (n_list + kTcDownK - 1) / kTcDownK;
+    float* ps = L.partial + (size_t)sl * L.batch * d;
+    const int q = warp & 3, col = n0 + 32 * q + lane;
+    if (nk == 0) {
+        // an empty slice still writes its partial (zeros)
+        for (int t = warp >> 2; t < L.batch; t += 2) ps[(size_t)t * d + col] = 0.0f;
+        return;
+    }
+    tc_setup<MT>(ts);
+    int piece = -1;  // list entries [piece * kTcDownPiece, +kTcDownPiece) of the slice are in pos[]
+    auto resolve = [&](int pc) {
+        __syncthreads();  // nobody reads the previous piece any more
+        const int e0 = k_begin + pc * kTcDownPiece;
+        const int e1 = min(k_end, e0 + kTcDownPiece);
+        for (int i = tid; i < kTcDownPiece; i += kGuThreads) pos[i] = -1;
+        __syncthreads();
+        bit_emit(ub, L.n_rows, bs, e0, e1, pos);
+        __syncthreads();
+        piece = pc;
+    };
+    auto load = [&](int kb, int stage) {
+        unsigned char* base = sm + stage * C::kStage;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            // W_down: 64 rows x 16 chunks of 8 columns
+            const int qq = tid + kGuThreads * i;
+            const int r = qq >> 4, c16 = qq & 15;
+            const int li = kb * kTcDownK + r;
+            const int pp = li < n_list ? pos[li - piece * kTcDownPiece] : -1;
+            const int j = pp >= 0 ? (L.rows ? L.rows[pp] : pp) : 0;
+            const int h = c16 >> 3, c = c16 & 7;
+            cp16(base + h * C::kAHalf + swz(r, c, 128), L.wd + (size_t)j * d + n0 + c16 * 8, pp >= 0);
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            // c hi / lo: 64 rows x 8 chunks of 8 tokens each
+            const int qq = tid + kGuThreads * i;
+            const int lo = qq >> 9, r = (qq >> 3) & 63, c = qq & 7;
+            const int li = kb * kTcDownK + r;
+            const int pp = li < n_list ? pos[li - piece * kTcDownPiece] : -1;
+            const size_t off = (size_t)(pp >= 0 ? pp : 0) * kTokPad + c * 8;
+            cp16(base + C::kA + lo * C::kC + swz(r, c, 128), (lo ? L.c_lo : L.c_hi) + off, pp >= 0);
+        }
+    };
+    auto ensure_piece = [&](int kb) {
+        const int pc = kb * kTcDownK / kTcDownPiece;
+        if (pc != piece) resolve(pc);
+    };
+    const uint32_t sm0 = smem_addr(sm);
+    constexpr int S = C::kStages, D = kMmaLag;
+    bool ok = true;
+    for (int s = 0; s < S - D; ++s) {
+        if (s < nk) {
+            ensure_piece(s);
+            load(s, s);
+        }
+        cp_commit();
+    }
+    for (int kb = 0; kb < nk; ++kb) {
+        cp_wait<S - D - 1>();
+        fence_proxy_async_smem();
+        __syncthreads();
+        if (ts.fail) {
+            ok = false;
+            break;
+        }
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t a0 = sm0 + (kb % S) * C::kStage;
+            const uint32_t b0 = a0 + C::kA;
+#pragma unroll
+            for (int kk = 0; kk < kTcDownK / 16; ++kk) {  // 16 rows = two 8-row atoms per MMA
+                const uint64_t ad = sdesc_mn128(a0 + kk * 2048, C::kAHalf);
+                tc_mma(ts.tmem, ad, sdesc_mn128(b0 + kk * 2048, C::kC), C::kIdesc, (kb | kk) != 0);
+                tc_mma(ts.tmem, ad, sdesc_mn128(b0 + C::kC + kk * 2048, C::kC), C::kIdesc, 1u);
+            }
+            tc_commit(&ts.mma_done[kb % S]);
+        }
+        const int nxt = kb + S - D;
+        if (nxt < nk) {
+            if (kb >= D && !mbar_wait(&ts.mma_done[(kb - D) % S], (unsigned)((kb - D) / S) & 1u)) ts.fail = 1;
+            ensure_piece(nxt);
+            load(nxt, nxt % S);
+        }
+        cp_commit();
+    }
+    if (ok && !mbar_wait(&ts.mma_done[(nk - 1) % S], (unsigned)((nk - 1) / S) & 1u)) ts.fail = 1;
+    cp_wait<0>();
+    __syncthreads();
+    ok = ok && ts.fail == 0;
+    if (!ok && tid == 0) atomicOr(L.status, kStatusTimeout);
+    tc_fence_after();
+    if (ok) {
+        // warp w: columns n0 + 32 (w % 4) + lane, token tiles w / 4, w / 4 + 2
+        for (int mt = warp >> 2; mt < MT; mt += 2) {
+            float v[16];
+            tc_ld16(ts.tmem + ((uint32_t)(32 * q) << 16) + 16 * mt, v);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int t = 16 * mt + e;
+                if (t < L.batch) ps[(size_t)t * d + col] = v[e];
+            }
+        }
+    }
+    tc_teardown<MT>(ts);
+}
+
 // y_t = sum of the slices' partials in slice order (or h_t += y_t)
 __global__ void __launch_bounds__(256) k_wide_reduce(const WideLaunch L) {
     pdl_wait();
@@ -665,13 +880,28 @@ cudaError_t launch(K kernel, int grid, int threads, size_t smem, cudaStream_t st
     return cudaLaunchKernelEx(&lc, kernel, L);
 }
 
+// The tensor-core down kernel (128-column tiles) for passes of more than 48
+// tokens; the mma.sync one (256-column tiles, half the c traffic per weight
+// byte) below that, where it measured faster.
+constexpr bool tc_down(int mt) { return mt >= 4; }
+
 template <int MT>
-cudaError_t run_t(const WideLaunch& L, cudaStream_t stream, bool pdl) {
+cudaError_t run_t(const WideLaunch& L0, cudaStream_t stream, bool pdl) {
+    WideLaunch L = L0;
+    // the tensor-core down kernel's column tiles are half as wide: half as
+    // many slices keep its grid at about one CTA per SM (the reduction sums
+    // the same count)
+    if (tc_down(MT)) L.ks = L0.ks * kTcDownCols / kDownCols > 0 ? L0.ks * kTcDownCols / kDownCols : 1;
     const int gu_grid = (L.n_rows + kTcRows - 1) / kTcRows;
     cudaError_t e = launch(k_wide_gate<MT>, gu_grid, kGuThreads, TcCfg<MT>::kBytes, stream, pdl, L);
     if (e == cudaSuccess) e = launch(k_wide_up<MT>, gu_grid, kGuThreads, TcCfg<MT>::kBytes, stream, true, L);
-    if (e == cudaSuccess)
-        e = launch(k_wide_down<MT>, (L.d / kDownCols) * L.ks, kDownThreads, DnSmem::kBytes, stream, true, L);
+    if (e == cudaSuccess) {
+        if (tc_down(MT))
+            e = launch(k_wide_down_tc<MT>, (L.d / kTcDownCols) * L.ks, kGuThreads, TcDownCfg<MT>::kBytes, stream,
+                       true, L);
+        else
+            e = launch(k_wide_down<MT>, (L.d / kDownCols) * L.ks, kDownThreads, DnSmem::kBytes, stream, true, L);
+    }
     if (e == cudaSuccess) {
         const int n = L.batch * L.d;
         e = launch(k_wide_reduce, (n + 255) / 256, 256, 0, stream, true, L);
@@ -684,6 +914,8 @@ cudaError_t prepare_t() {
     cudaError_t e = cudaFuncSetAttribute(k_wide_gate<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<MT>::kBytes);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_wide_up<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<MT>::kBytes);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_wide_down<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, DnSmem::kBytes);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_wide_down_tc<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcDownCfg<MT>::kBytes);
     return e;
 }
 
@@ -694,6 +926,7 @@ bool wide_supported(int wdtype, int d, int m, int batch) {
 }
 
 int wide_slices(int d, int num_sms) {
+    // enough slices for either down kernel (the tensor-core one has narrower column tiles)
     const int n_tiles = d / kDownCols;
     return n_tiles >= num_sms ? 1 : num_sms / n_tiles;
 }
