@@ -1104,17 +1104,18 @@ static size_t mma_smem(int d, MmaCfg* mc) {
 constexpr int kQ4Rows = 4;          // rows per subtask
 constexpr int kQ4SlotsPerWarp = 2;  // ring slots per consumer warp
 constexpr int kQ4QuarterPad = 16;   // bytes after each K-quarter of an activation row
+// bytes of the activations' 32-element group sums (kAccMaxTokens rows)
+__host__ __device__ constexpr size_t q4_xsum_bytes(int d) {
+    return ((size_t)kAccMaxTokens * (d / 32) * sizeof(float) + 127) / 128 * 128;
+}
 
 // bf16x2 A-fragment register of two INT4 codes held at bits 0-3 and 16-19
-// of v: (code_lo - 8, code_hi - 8), exact. 0x4300 is 128.0 in bf16, whose
-// last mantissa bit is worth 1.0, so OR-ing a code into it gives 128 + code;
-// subtracting 136 leaves code - 8.
-__device__ __forceinline__ uint32_t q4_frag(uint32_t v) {
-    const uint32_t b = (v & 0x000F000Fu) | 0x43004300u;
-    __nv_bfloat162 p = *reinterpret_cast<const __nv_bfloat162*>(&b);
-    p = __hsub2(p, __floats2bfloat162_rn(136.0f, 136.0f));
-    return *reinterpret_cast<const uint32_t*>(&p);
-}
+// of v: (128 + code_lo, 128 + code_hi), exact. 0x4300 is 128.0 in bf16,
+// whose last mantissa bit is worth 1.0, so OR-ing a code into it gives
+// 128 + code. The dequantized weight is code - 8: a group's dot product with
+// these pairs is corrected afterwards by 136 times the group's activation
+// sum, one fma per group instead of a subtraction per pair.
+__device__ __forceinline__ uint32_t q4_frag(uint32_t v) { return (v & 0x000F000Fu) | 0x43004300u; }
 // d += A * B for one m16n8k16 step with all 16 A rows.
 __device__ __forceinline__ void mma_bf16_16816_a4(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
                                                   uint32_t b0, uint32_t b1) {
@@ -1147,8 +1148,8 @@ __device__ __forceinline__ void cp_async_wait() {
 
 template <int NT, typename Stage>
 __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char* ring, const unsigned char* xb,
-                            ChunkState<NT>* tab, const MmaCfg& mc, int i0, int i1, int n_chunks, int cidx,
-                            int lane, Stage stage) {
+                            const float* xsum, ChunkState<NT>* tab, const MmaCfg& mc, int i0, int i1, int n_chunks,
+                            int cidx, int lane, Stage stage) {
     constexpr int C = GateUpWarps<NT>::C;
     const int cthreads = C * kWarp;
     const int d = a.d;
@@ -1172,6 +1173,8 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
     // and their products are not used
     const int n = lane % 8;
     const int n_tok = NT > 1 ? n / 4 : 0;
+    // activation sums of the groups of this lane's product (token t / 2)
+    const float* xg = xsum + (NT > 1 ? t / 2 : 0) * (d / 32) + qu * nq;
     const int n_q = (n & 1) ? 2 + ((n >> 1) & 1) : ((n >> 1) & 1);
     const uint32_t x_col = smem_u32(xb) + n_tok * mc.x_stride + n_q * (d / 2 + kQ4QuarterPad) + (lane / 8) * 16;
     const uint32_t x_step = 64u;
@@ -1209,6 +1212,9 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
             const float2 sc = __half22float2(*reinterpret_cast<const __half2*>(sp + G * 2));
             const float s0 = (qu & 1) ? sc.y : sc.x;
             const float s1 = (qu & 1) ? sc.x : sc.y;
+            const float2 xs = *reinterpret_cast<const float2*>(xg + G);
+            const float x0 = (qu & 1) ? xs.y : xs.x;
+            const float x1 = (qu & 1) ? xs.x : xs.y;
             uint32_t cw[4];  // (qa, G), (qb, G), (qa, G + 1), (qb, G + 1) in this lane's order
             ldsm_x4(c_addr + G * 16, cw[0], cw[1], cw[2], cw[3]);
 #pragma unroll
@@ -1224,11 +1230,12 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
                 mma_bf16_16816_a4(dg, q4_frag(ca), q4_frag(cb), q4_frag(ca >> 4), q4_frag(cb >> 4), b0, b1);
                 mma_bf16_16816_a4(dh, q4_frag(ca >> 8), q4_frag(cb >> 8), q4_frag(ca >> 12), q4_frag(cb >> 12), b0n,
                                   b1n);
+                // sum over the group of (128 + code) x, less 136 times the sum of x
                 const float pv = use_d0 ? dg[0] + dh[0] : dg[3] + dh[3];
                 if (h == 0)
-                    v0 = fmaf(s0, pv, v0);
+                    v0 = fmaf(s0, fmaf(-136.0f, x0, pv), v0);
                 else
-                    v1 = fmaf(s1, pv, v1);
+                    v1 = fmaf(s1, fmaf(-136.0f, x1, pv), v1);
             }
         }
         // the four K-quarters of (row wr, token t / 2), in the same order in every lane
@@ -1411,10 +1418,12 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
     constexpr int C = GateUpWarps<NT>::C;
     __shared__ GateUpShared<NT> sh;
     extern __shared__ __align__(128) unsigned char dyn[];
-    // [NT][4 quarters][d/4 bf16 + pad] activations, the ring, the round's chunks
+    // [NT][4 quarters][d/4 bf16 + pad] activations, their group sums, the
+    // ring, the round's chunks
     unsigned char* xb = dyn;
     const size_t x_bytes = ((size_t)kAccMaxTokens * mc.x_stride + 127) / 128 * 128;
-    unsigned char* ring = dyn + x_bytes;  // [C][2 slots][kQ4Rows][w_stride]
+    float* xsum = reinterpret_cast<float*>(dyn + x_bytes);  // [NT][d/32]
+    unsigned char* ring = dyn + x_bytes + q4_xsum_bytes(a.d);  // [C][2 slots][kQ4Rows][w_stride]
     ChunkState<NT>* tab = reinterpret_cast<ChunkState<NT>*>(ring + (size_t)mc.groups * kQ4Rows * mc.w_stride);
     const int n_x = a.route ? a.batch : a.nt;
 
@@ -1440,7 +1449,8 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
     const int cthreads = C * kWarp;
     const int x_tok0 = a.route ? 0 : a.tok0;
     const int dq = a.d / 4;
-    auto xpos = [&](int i) { return (i / dq) * (dq + kQ4QuarterPad / 2) + i % dq; };  // bf16 index in a row
+    // bf16 index in a row of element i (i < d): K-quarter (i >= dq) + (i >= 2dq) + (i >= 3dq)
+    auto xpos = [&](int i) { return i + ((i >= dq) + (i >= 2 * dq) + (i >= 3 * dq)) * (kQ4QuarterPad / 2); };
     // Stage the activations; first_rows() (the first weight-row copies) runs
     // once, right after the first activation loads are issued.
     auto stage = [&](auto&& first_rows) {
@@ -1464,8 +1474,29 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
         }
         once();
         named_bar_sync(1, cthreads);
+        // each 32-element group's sum of the staged activations, in order
+        const int ng = a.d / 32;
+        for (int i = ctid; i < NT * ng; i += cthreads) {
+            const int t = i / ng;
+            const __nv_bfloat16* xr =
+                reinterpret_cast<const __nv_bfloat16*>(xb + (size_t)t * mc.x_stride) + xpos((i - t * ng) * 32);
+            float sum = 0.0f;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const uint4 v = *reinterpret_cast<const uint4*>(xr + 8 * k);
+                const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float2 f = __bfloat1622float2(p[q]);
+                    sum += f.x;
+                    sum += f.y;
+                }
+            }
+            xsum[i] = sum;
+        }
+        named_bar_sync(1, cthreads);
     };
-    consume_q4w<NT>(a, sh, ring, xb, tab, mc, i0, i1, n_chunks, warp - 1, lane, stage);
+    consume_q4w<NT>(a, sh, ring, xb, xsum, tab, mc, i0, i1, n_chunks, warp - 1, lane, stage);
     down_partial<T, NT, true>(a, sh, i0, i1, n_chunks, warp - 1, lane);
 }
 
@@ -1484,7 +1515,7 @@ static size_t q4w_smem(int d, int avail, MmaCfg* mc) {
     mc->lookahead = 0;
     mc->end_tasks = 0;
     (void)avail;
-    return x_bytes + (size_t)mc->groups * slot + (size_t)kQ4Round * sizeof(ChunkState<kAccMaxTokens>);
+    return x_bytes + q4_xsum_bytes(d) + (size_t)mc->groups * slot + (size_t)kQ4Round * sizeof(ChunkState<kAccMaxTokens>);
 }
 
 // ---------------------------------------------------------------------------

@@ -386,7 +386,8 @@ __device__ __forceinline__ void stage_act_row(const float* __restrict__ h, const
         float tot = 0.0f;
         for (int w = 0; w < nw; ++w) tot += red[w];
         const float rms = __fsqrt_rn(__fadd_rn(__fdiv_rn(tot, (float)d), 1e-5f));
-        auto norm = [&](int i, float hv) { return (i == d - 1) ? 1.0f : Vec<T>::round_act(__fdiv_rn(hv, rms)); };
+        const float rinv = __frcp_rn(rms);  // one reciprocal, then a product per element
+        auto norm = [&](int i, float hv) { return (i == d - 1) ? 1.0f : Vec<T>::round_act(__fmul_rn(hv, rinv)); };
         const bool kept = d4 <= group;  // the single group is still in registers
         for (int g0 = 0; g0 < d4; g0 += group) {
 #pragma unroll
