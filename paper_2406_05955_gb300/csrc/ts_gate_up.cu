@@ -426,12 +426,11 @@ __device__ __forceinline__ void partial_blocks_q4(const FfnLaunch& a, GateUpShar
     }
 }
 
-template <typename T, int NT, bool Q4 = false>
+template <typename T, int NT, bool Q4 = false, int C = GateUpWarps<NT>::C>
 __device__ void down_partial(const FfnLaunch& a, GateUpShared<NT>& sh, int i0, int i1, int n_chunks, int cidx,
                              int lane) {
     constexpr int VEC = Vec<T>::N;
     constexpr int BLK = kWarp * VEC;
-    constexpr int C = GateUpWarps<NT>::C;
     constexpr int AT = kAccMaxTokens;
     const int cthreads = C * kWarp;
     const int d = a.d;
@@ -1102,6 +1101,7 @@ static size_t mma_smem(int d, MmaCfg* mc) {
 // swapped order, which keeps the lanes' shared-memory words in distinct banks.
 // ---------------------------------------------------------------------------
 constexpr int kQ4Rows = 4;          // rows per subtask
+constexpr int kQ4Consumers = 8;     // consumer warps (10 fit in shared memory but measured no faster)
 constexpr int kQ4SlotsPerWarp = 2;  // ring slots per consumer warp
 constexpr int kQ4QuarterPad = 16;   // bytes after each K-quarter of an activation row
 // bytes of the activations' 32-element group sums (kAccMaxTokens rows)
@@ -1150,7 +1150,7 @@ template <int NT, typename Stage>
 __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char* ring, const unsigned char* xb,
                             const float* xsum, ChunkState<NT>* tab, const MmaCfg& mc, int i0, int i1, int n_chunks,
                             int cidx, int lane, Stage stage) {
-    constexpr int C = GateUpWarps<NT>::C;
+    constexpr int C = kQ4Consumers;
     const int cthreads = C * kWarp;
     const int d = a.d;
     const int nq = d / 128;  // 32-element groups per K-quarter
@@ -1207,7 +1207,7 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
         const uint32_t c_addr = smem_u32(sbase + (size_t)(lg % 4) * mc.w_stride + l_off);
         const unsigned char* sp = row + d / 2 + qu * nq * 2;  // binary16 scales of quarter qu
         float v0 = 0.0f, v1 = 0.0f;
-#pragma unroll 2
+#pragma unroll 4
         for (int G = 0; G < nq; G += 2) {
             const float2 sc = __half22float2(*reinterpret_cast<const __half2*>(sp + G * 2));
             const float s0 = (qu & 1) ? sc.y : sc.x;
@@ -1413,9 +1413,9 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
 }
 
 template <int NT>
-__global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(const FfnLaunch a, const MmaCfg mc) {
+__global__ void __launch_bounds__((kQ4Consumers + 1) * kWarp, 1) k_gate_up_q4w(const FfnLaunch a, const MmaCfg mc) {
     using T = __nv_bfloat16;  // activations
-    constexpr int C = GateUpWarps<NT>::C;
+    constexpr int C = kQ4Consumers;
     __shared__ GateUpShared<NT> sh;
     extern __shared__ __align__(128) unsigned char dyn[];
     // [NT][4 quarters][d/4 bf16 + pad] activations, their group sums, the
@@ -1497,7 +1497,7 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_q4w(con
         named_bar_sync(1, cthreads);
     };
     consume_q4w<NT>(a, sh, ring, xb, xsum, tab, mc, i0, i1, n_chunks, warp - 1, lane, stage);
-    down_partial<T, NT, true>(a, sh, i0, i1, n_chunks, warp - 1, lane);
+    down_partial<T, NT, true, kQ4Consumers>(a, sh, i0, i1, n_chunks, warp - 1, lane);
 }
 
 // Shared memory of the INT4 kernel: activations (kAccMaxTokens rows of four
@@ -1509,7 +1509,7 @@ static size_t q4w_smem(int d, int avail, MmaCfg* mc) {
     mc->x_stride = 4 * (d / 2 + kQ4QuarterPad);
     mc->w_stride = row_bytes + ((32 - row_bytes % 128) % 128 + 128) % 128;
     const size_t x_bytes = ((size_t)kAccMaxTokens * mc->x_stride + 127) / 128 * 128;
-    const int C = GateUpWarps<1>::C;
+    const int C = kQ4Consumers;
     const size_t slot = (size_t)kQ4Rows * mc->w_stride;
     mc->groups = C * kQ4SlotsPerWarp;
     mc->lookahead = 0;
@@ -2085,7 +2085,7 @@ static cudaError_t launch_q4w_t(const FfnLaunch& a, int grid, cudaStream_t strea
     if (smem + kSmemMargin > (size_t)g_optin) return cudaErrorInvalidValue;
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(grid);
-    lc.blockDim = dim3(GateUpWarps<NT>::THREADS);
+    lc.blockDim = dim3((kQ4Consumers + 1) * kWarp);
     lc.dynamicSmemBytes = smem;
     lc.stream = stream;
     cudaLaunchAttribute attr[1];
