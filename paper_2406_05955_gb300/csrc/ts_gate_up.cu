@@ -179,21 +179,28 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, unsigned parity, int la
     return __shfl_sync(0xffffffffu, ok, 0) != 0;
 }
 
-// Write a finished chunk's outputs (warp-wide) and free its window slot:
-// per-token gate/both bitmap bytes, union bytes, and c by batch slot.
+// Write finished chunks' outputs: per-token gate/both bitmap bytes, union
+// bytes, and c by batch slot. One warp takes up to kWarp / kChunk chunks at
+// once, chunk tab[c0 + q] in lanes 8q .. 8q + 7 (lane 8q + r holds its row r),
+// so the chunk states are read in parallel instead of one chunk after another.
+constexpr int kFinPerWarp = kWarp / kChunk;
 template <int NT>
-__device__ void finalize_chunk_s(const FfnLaunch& a, GateUpShared<NT>& sh, volatile ChunkState<NT>& s, int lane) {
+__device__ void finalize_chunks(const FfnLaunch& a, GateUpShared<NT>& sh, volatile ChunkState<NT>* tab, int c0,
+                                int nc, int lane) {
+    const int q = lane / kChunk, r = lane % kChunk;
+    const bool on = q < nc;
+    volatile ChunkState<NT>& s = tab[c0 + (on ? q : 0)];
     const int e = s.e;
     const int chunk = s.chunk;
     const int ntok = sh.es.ntok[e];
     const unsigned gm = s.gmask;
-    const int j = lane < kChunk ? s.jr[lane] : -1;
-    const bool up_row = lane < kChunk && ((gm >> lane) & 1u);
+    const int j = on ? s.jr[r] : -1;
+    const bool up_row = on && ((gm >> r) & 1u);
     float g[NT], u[NT];
 #pragma unroll
     for (int k = 0; k < NT; ++k) {
-        g[k] = lane < kChunk ? s.g[lane][k] : 0.0f;
-        u[k] = up_row ? s.u[lane][k] : 0.0f;
+        g[k] = on ? s.g[r][k] : 0.0f;
+        u[k] = up_row ? s.u[r][k] : 0.0f;
     }
     unsigned ub = 0u;
     uint8_t* gb = a.gbits + (size_t)e * a.bits_expert_stride + chunk;
@@ -203,30 +210,32 @@ __device__ void finalize_chunk_s(const FfnLaunch& a, GateUpShared<NT>& sh, volat
     for (int k = 0; k < NT; ++k) {
         const bool gk = j >= 0 && g[k] > 0.0f;
         both[k] = gk && up_row && u[k] > 0.0f;
+        // this lane's group's byte of the warp-wide ballots
+        const unsigned gbyte = (__ballot_sync(0xffffffffu, gk) >> (kChunk * q)) & 0xffu;
+        const unsigned bbyte = (__ballot_sync(0xffffffffu, both[k]) >> (kChunk * q)) & 0xffu;
         if (k < ntok) {
-            const unsigned gbyte = __ballot_sync(0xffffffffu, gk) & 0xffu;
-            const unsigned bbyte = __ballot_sync(0xffffffffu, both[k]) & 0xffu;
             ub |= bbyte;
-            if (lane == 0) {
+            if (on && r == 0) {
                 const size_t tb = (size_t)(a.bits_tok_base + k) * a.nbytes;
                 gb[tb] = (uint8_t)gbyte;
                 bb[tb] = (uint8_t)bbyte;
             }
         }
     }
-    if (lane == 0) {
+    if (on && r == 0) {
         a.ubits[(size_t)e * a.nbytes + chunk] = (uint8_t)ub;
         a.ugbits[(size_t)e * a.nbytes + chunk] = (uint8_t)gm;
     }
+    const bool b_row = on && ((ub >> r) & 1u);
     // The down projection will gather these W_down rows: pull them into L2
     // now, while HBM is streaming anyway.
-    if (lane < kChunk && ((ub >> lane) & 1u))
+    if (b_row)
         prefetch_l2_bulk(static_cast<const unsigned char*>(a.ex[e].wd) + (size_t)j * a.row_bytes,
                          (unsigned)a.row_bytes);
     // c by batch slot: the pass-local token (single FFN) or the global token
     // (MoE, 0 for tokens not routed to this expert)
-    if (lane < kChunk && ((ub >> lane) & 1u)) {
-        float* cv = a.cval + ((size_t)e * kMaxPass) * a.cval_tok_stride + (size_t)chunk * kChunk + lane;
+    if (b_row) {
+        float* cv = a.cval + ((size_t)e * kMaxPass) * a.cval_tok_stride + (size_t)chunk * kChunk + r;
         float val[NT];
 #pragma unroll
         for (int k = 0; k < NT; ++k) val[k] = (k < ntok && both[k]) ? sh.es.w[e][k] * (g[k] * u[k]) : 0.0f;
@@ -245,20 +254,18 @@ __device__ void finalize_chunk_s(const FfnLaunch& a, GateUpShared<NT>& sh, volat
         }
     }
     if constexpr (NT <= kAccMaxTokens) {
-        const int q = s.q;
-        if (q < kMaxLocal) {
-            if (lane == 0) sh.pd.ub[q] = (uint8_t)ub;
-            if (lane < kChunk) {
+        const int ql = s.q;
+        if (on && ql < kMaxLocal) {
+            if (r == 0) sh.pd.ub[ql] = (uint8_t)ub;
 #pragma unroll
-                for (int t = 0; t < kAccMaxTokens; ++t) {
-                    float v = 0.0f;
+            for (int t = 0; t < kAccMaxTokens; ++t) {
+                float v = 0.0f;
 #pragma unroll
-                    for (int k = 0; k < NT; ++k) {
-                        const int slot_of_k = a.route ? sh.es.tok[e][k] : k;
-                        if (k < ntok && both[k] && slot_of_k == t) v = sh.es.w[e][k] * (g[k] * u[k]);
-                    }
-                    sh.pd.c[q][lane][t] = v;
+                for (int k = 0; k < NT; ++k) {
+                    const int slot_of_k = a.route ? sh.es.tok[e][k] : k;
+                    if (k < ntok && both[k] && slot_of_k == t) v = sh.es.w[e][k] * (g[k] * u[k]);
                 }
+                sh.pd.c[ql][r][t] = v;
             }
         }
     }
@@ -266,7 +273,7 @@ __device__ void finalize_chunk_s(const FfnLaunch& a, GateUpShared<NT>& sh, volat
 }
 template <int NT>
 __device__ void finalize_chunk(const FfnLaunch& a, GateUpShared<NT>& sh, int cw, int lane) {
-    finalize_chunk_s<NT>(a, sh, sh.cs[cw], lane);
+    finalize_chunks<NT>(a, sh, sh.cs, cw, 1, lane);
     __threadfence_block();
     if (lane == 0) mbar_arrive(&sh.chunk_free[cw]);
 }
@@ -1407,7 +1414,8 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
             }
             if (phase == 0) named_bar_sync(1, cthreads);
         }
-        for (int c = cidx; c < nr; c += C) finalize_chunk_s<NT>(a, sh, tab[c], lane);
+        for (int c0 = cidx * kFinPerWarp; c0 < nr; c0 += C * kFinPerWarp)
+            finalize_chunks<NT>(a, sh, tab, c0, min(kFinPerWarp, nr - c0), lane);
         named_bar_sync(1, cthreads);  // the table is refilled next round
     }
 }
@@ -1722,7 +1730,8 @@ __device__ void consume_rows(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned 
             }
             if (phase == 0) named_bar_sync(1, cthreads);
         }
-        for (int c = cidx; c < nr; c += C) finalize_chunk_s<NT>(a, sh, tab[c], lane);
+        for (int c0 = cidx * kFinPerWarp; c0 < nr; c0 += C * kFinPerWarp)
+            finalize_chunks<NT>(a, sh, tab, c0, min(kFinPerWarp, nr - c0), lane);
         named_bar_sync(1, cthreads);  // the table is refilled next round
     }
 }
