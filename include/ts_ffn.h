@@ -46,7 +46,8 @@ typedef enum {
     TS_ERR_OOM = 3,          /* scratch allocation failed                    */
     TS_ERR_BAD_INDEX = 4,    /* the GPU saw an out-of-range/unsorted list    */
     TS_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up           */
-    TS_ERR_UNSUPPORTED = 6   /* valid request this build does not handle     */
+    TS_ERR_UNSUPPORTED = 6,  /* valid request this build does not handle     */
+    TS_ERR_SCRATCH = 7       /* a scratch guard zone was overwritten         */
 } ts_status;
 
 /*
@@ -163,6 +164,20 @@ ts_status ts_ffn_get_active(ts_ffn* h, cudaStream_t stream, int token, int32_t* 
 ts_status ts_ffn_get_error(ts_ffn* h, cudaStream_t stream);
 
 /*
+ * Scratch guard check (a debugging aid, not part of the method). Every block
+ * of a handle's device scratch (partial sums, bitmaps, c values, status
+ * word, ...) is followed by a guard zone filled with one byte value when the
+ * handle is created. This call synchronises `stream` and compares every zone
+ * with its fill: TS_OK if all are intact, TS_ERR_SCRATCH if a kernel wrote
+ * past the end of a block, TS_ERR_INVALID_ARG for a NULL handle.
+ * ts_ffn_poke_guard overwrites one byte of guard zone i (0 <= i < the number
+ * of blocks; TS_ERR_INVALID_ARG otherwise) from the host, so that a test can
+ * check that the check fires; the handle stays usable.
+ */
+ts_status ts_ffn_check_scratch(ts_ffn* h, cudaStream_t stream);
+ts_status ts_ffn_poke_guard(ts_ffn* h, int i);
+
+/*
  * Test hook for the failure-detection path (not part of the method): while
  * `on` is nonzero, forwards on this handle make one consumer warp of every
  * gate+up CTA wait on a barrier that nothing arrives at. The wait, like every
@@ -243,6 +258,9 @@ ts_status ts_moe_get_active(ts_moe* h, cudaStream_t stream, int expert, int toke
 /* As ts_ffn_get_error, for the MoE layer's router and grouped kernels. */
 ts_status ts_moe_get_error(ts_moe* h, cudaStream_t stream);
 
+/* As ts_ffn_check_scratch, for the MoE layer's scratch. */
+ts_status ts_moe_check_scratch(ts_moe* h, cudaStream_t stream);
+
 /*
  * Activation predictor of one FFN layer (Sec. 7: a predictor per FFN block,
  * per expert for MoE; the paper gives no architecture, so this is a reading):
@@ -267,6 +285,9 @@ ts_status ts_moe_get_error(ts_moe* h, cudaStream_t stream);
 ts_status ts_predictor_create(ts_predictor** out, int d, int r, int m, ts_dtype dtype, const void* w1,
                               const void* w2, int max_batch);
 void ts_predictor_destroy(ts_predictor* p);
+
+/* As ts_ffn_check_scratch, for the predictor's scratch. */
+ts_status ts_predictor_check_scratch(ts_predictor* p, cudaStream_t stream);
 
 /*
  * list[0..K) = the predicted neurons for the batch x [batch][d] (device,

@@ -15,10 +15,14 @@ import numpy as np
 import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "_build", "libtsffn.so")
+# TS_FFN_DEBUG=1 in the environment loads the debug build instead (the same
+# kernels with every gathered row index range-checked into the status word).
+_DEBUG = os.environ.get("TS_FFN_DEBUG", "") == "1"
+LIB_PATH = os.path.join(_HERE, "_build", "debug", "libtsffn_debug.so") if _DEBUG else \
+    os.path.join(_HERE, "_build", "libtsffn.so")
 
 TS_OK, TS_ERR_INVALID_ARG, TS_ERR_CUDA, TS_ERR_OOM, TS_ERR_BAD_INDEX, TS_ERR_TIMEOUT, \
-    TS_ERR_UNSUPPORTED = range(7)
+    TS_ERR_UNSUPPORTED, TS_ERR_SCRATCH = range(8)
 TS_F32, TS_BF16, TS_INT4 = 0, 1, 2
 
 _lock = threading.Lock()
@@ -42,6 +46,8 @@ SIGNATURES = {
     "ts_stack_forward": (I, [P, I, P, I, P, P, P]),
     "ts_ffn_get_active": (I, [P, P, I, P, IP, P, IP]),
     "ts_ffn_get_error": (I, [P, P]),
+    "ts_ffn_check_scratch": (I, [P, P]),
+    "ts_ffn_poke_guard": (I, [P, I]),
     "ts_ffn_set_test_stall": (I, [P, I]),
     "ts_ffn_forward_noalloc": (I, [I, I, I, P, P, P, P, I, P, P, P, I]),
     "ts_moe_create": (I, [PP, I, I, I, I, P, P, I]),
@@ -51,11 +57,13 @@ SIGNATURES = {
     "ts_moe_get_routing": (I, [P, P, P, P]),
     "ts_moe_get_active": (I, [P, P, I, I, P, IP, P, IP]),
     "ts_moe_get_error": (I, [P, P]),
+    "ts_moe_check_scratch": (I, [P, P]),
     "ts_graph_capture_stack": (I, [PP, P, I, P, I, P, P]),
     "ts_graph_capture_stack_fused": (I, [PP, P, I, P, I, P, P]),
     "ts_graph_capture_moe_stack": (I, [PP, P, I, P, I]),
     "ts_predictor_create": (I, [PP, I, I, I, I, P, P, I]),
     "ts_predictor_destroy": (None, [P]),
+    "ts_predictor_check_scratch": (I, [P, P]),
     "ts_predict": (I, [P, P, I, I, P, P, P]),
     "ts_stack_forward_predicted": (I, [P, P, I, P, I, P, P, P]),
     "ts_graph_capture_stack_predicted": (I, [PP, P, P, I, P, I, P, P]),
@@ -233,6 +241,14 @@ class Ffn:
     def get_error(self, stream=None) -> int:
         return int(lib().ts_ffn_get_error(self.handle, _stream(stream)))
 
+    def check_scratch(self, stream=None) -> int:
+        """Status of the scratch guard zones: TS_OK, or TS_ERR_SCRATCH if one was overwritten."""
+        return int(lib().ts_ffn_check_scratch(self.handle, _stream(stream)))
+
+    def poke_guard(self, i: int) -> None:
+        """Test hook: overwrite one byte of scratch guard zone ``i`` from the host."""
+        _check(lib().ts_ffn_poke_guard(self.handle, int(i)), "ts_ffn_poke_guard")
+
     def set_test_stall(self, on: bool) -> None:
         """Failure-detection test hook: the next forwards' bounded waits run out."""
         _check(lib().ts_ffn_set_test_stall(self.handle, int(bool(on))), "ts_ffn_set_test_stall")
@@ -355,6 +371,10 @@ class Predictor:
                                 _stream(stream)), "ts_predict")
         return out[: int(K)]
 
+    def check_scratch(self, stream=None) -> int:
+        """Status of the scratch guard zones (as Ffn.check_scratch)."""
+        return int(lib().ts_predictor_check_scratch(self.handle, _stream(stream)))
+
     def close(self) -> None:
         if getattr(self, "_h", None) is not None:
             lib().ts_predictor_destroy(self._h)
@@ -448,6 +468,10 @@ class Moe:
 
     def get_error(self, stream=None) -> int:
         return int(lib().ts_moe_get_error(self.handle, _stream(stream)))
+
+    def check_scratch(self, stream=None) -> int:
+        """Status of the scratch guard zones (as Ffn.check_scratch)."""
+        return int(lib().ts_moe_check_scratch(self.handle, _stream(stream)))
 
     def close(self) -> None:
         if getattr(self, "_h", None) is not None:

@@ -19,6 +19,10 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libtsffn.so")
+# The same sources with -DTS_DEBUG: every gathered row index is range-checked
+# into the status word (see debug_row in csrc/ts_kernels.cuh).
+DEBUG_DIR = os.path.join(OUT_DIR, "debug")
+DEBUG_LIB = os.path.join(DEBUG_DIR, "libtsffn_debug.so")
 SOURCES = ["ts_api.cu", "ts_gate_up.cu", "ts_down.cu", "ts_router.cu", "ts_noalloc.cu", "ts_wide.cu",
            "ts_topk.cu", "ts_predict.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -39,38 +43,54 @@ def _inputs() -> list[str]:
     return files + [os.path.abspath(__file__)]
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+def up_to_date(lib: str = LIB) -> bool:
+    if not os.path.exists(lib):
         return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(f) <= t for f in _inputs())
 
 
-def build(force: bool = False, verbose: bool = False, extra: list[str] | None = None) -> str:
-    """Compile and link libtsffn.so if any input changed; return its path."""
-    if not force and up_to_date():
-        return LIB
-    os.makedirs(OUT_DIR, exist_ok=True)
+def _build_libs(targets: list[tuple[str, str, list[str]]], verbose: bool) -> None:
+    """Compile every (library, object dir, extra flags) target's sources in one pool, then link each."""
     cc = nvcc()
-    flags = NVCC_FLAGS + (extra or [])
+    jobs = []
+    for lib, odir, flags in targets:
+        os.makedirs(odir, exist_ok=True)
+        jobs += [(src, odir, flags) for src in SOURCES]
 
-    def compile_one(src: str) -> str:
-        obj = os.path.join(OUT_DIR, src.replace(".cu", ".o"))
-        cmd = [cc, *ARCH, *flags, "-c", os.path.join(CSRC, src), "-o", obj]
+    def compile_one(job) -> str:
+        src, odir, flags = job
+        obj = os.path.join(odir, src.replace(".cu", ".o"))
+        cmd = [cc, *ARCH, *NVCC_FLAGS, *flags, "-c", os.path.join(CSRC, src), "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
-            raise RuntimeError(f"nvcc failed on {src}:\n{r.stderr}")
+            raise RuntimeError(f"nvcc failed on {src} ({' '.join(flags)}):\n{r.stderr}")
         if verbose and r.stderr:
             sys.stderr.write(r.stderr)
         return obj
 
-    with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        objs = list(ex.map(compile_one, SOURCES))
-    tmp = LIB + f".tmp{os.getpid()}"
-    r = subprocess.run([cc, *ARCH, "-shared", "-o", tmp, *objs], capture_output=True, text=True)
-    if r.returncode != 0:
-        raise RuntimeError(f"nvcc link failed:\n{r.stderr}")
-    os.replace(tmp, LIB)
+    with cf.ThreadPoolExecutor(max_workers=min(len(jobs), max(os.cpu_count() or 1, len(SOURCES)))) as ex:
+        objs = list(ex.map(compile_one, jobs))
+    for k, (lib, _, _) in enumerate(targets):
+        tmp = lib + f".tmp{os.getpid()}"
+        mine = objs[k * len(SOURCES):(k + 1) * len(SOURCES)]
+        r = subprocess.run([cc, *ARCH, "-shared", "-o", tmp, *mine], capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc link failed:\n{r.stderr}")
+        os.replace(tmp, lib)
+
+
+def build(force: bool = False, verbose: bool = False, extra: list[str] | None = None,
+          debug: bool = True) -> str:
+    """Compile and link libtsffn.so (and, with ``debug``, the range-checked
+    libtsffn_debug.so) if any input changed; return the release library's path."""
+    targets = []
+    if force or not up_to_date(LIB):
+        targets.append((LIB, OUT_DIR, list(extra or [])))
+    if debug and (force or not up_to_date(DEBUG_LIB)):
+        targets.append((DEBUG_LIB, DEBUG_DIR, ["-DTS_DEBUG", *(extra or [])]))
+    if targets:
+        _build_libs(targets, verbose)
     return LIB
 
 

@@ -1,7 +1,9 @@
 // ts_api.cu -- the C ABI of libtsffn (declared in include/ts_ffn.h): handles,
 // scratch arenas, argument validation, pass splitting, launch sequencing
 // with programmatic dependent launch, active-set export and graph capture.
+#include <nvtx3/nvToolsExt.h>
 #include <stdint.h>
+#include <stdio.h>
 #include <string.h>
 
 #include <algorithm>
@@ -55,12 +57,38 @@ ts_status device_info(DeviceInfo* di) {
 }
 
 // Carves sub-buffers out of one device allocation.
+// One NVTX range per layer of the stack calls, so that a profiler's timeline
+// shows the layers (header-only NVTX: with no tool attached the calls return
+// at once). The ranges are host-side: inside a stream capture they mark the
+// capture, not the graph's replays.
+struct LayerRange {
+    LayerRange(const char* what, int l) {
+        char name[64];
+        snprintf(name, sizeof name, "%s layer %d", what, l);
+        nvtxRangePushA(name);
+    }
+    ~LayerRange() { nvtxRangePop(); }
+    LayerRange(const LayerRange&) = delete;
+    LayerRange& operator=(const LayerRange&) = delete;
+};
+
+// A handle's device scratch: blocks carved out of one allocation. Every block
+// is followed by a guard zone of kGuardBytes filled with kGuardByte when the
+// arena is allocated; check_arena reads the zones back, so a kernel that
+// writes past the end of a scratch block is caught by the tests instead of
+// silently corrupting the next block.
+constexpr size_t kGuardBytes = kAlign;
+constexpr unsigned char kGuardByte = 0xA5;
+
 struct Arena {
     size_t bytes = 0;
     char* base = nullptr;
+    std::vector<size_t> guards;  // offsets of the guard zones
     size_t take(size_t n) {
         const size_t off = bytes;
         bytes += align_up(n);
+        guards.push_back(bytes);
+        bytes += kGuardBytes;
         return off;
     }
     template <typename P>
@@ -73,10 +101,26 @@ ts_status alloc_arena(Arena* ar) {
         ar->base = nullptr;
         return TS_ERR_OOM;
     }
-    if (cudaMemset(ar->base, 0, ar->bytes) != cudaSuccess) {
+    bool ok = cudaMemset(ar->base, 0, ar->bytes) == cudaSuccess;
+    for (size_t g : ar->guards) ok = ok && cudaMemset(ar->base + g, kGuardByte, kGuardBytes) == cudaSuccess;
+    if (!ok) {
         cudaFree(ar->base);
         ar->base = nullptr;
         return TS_ERR_CUDA;
+    }
+    return TS_OK;
+}
+
+// Synchronise `stream` and compare every guard zone with its fill.
+ts_status check_arena(const Arena& ar, cudaStream_t stream) {
+    if (!ar.base) return TS_ERR_INVALID_ARG;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return TS_ERR_CUDA;
+    std::vector<unsigned char> buf(kGuardBytes);
+    for (size_t g : ar.guards) {
+        if (cudaMemcpy(buf.data(), ar.base + g, kGuardBytes, cudaMemcpyDeviceToHost) != cudaSuccess)
+            return TS_ERR_CUDA;
+        for (unsigned char b : buf)
+            if (b != kGuardByte) return TS_ERR_SCRATCH;
     }
     return TS_OK;
 }
@@ -166,6 +210,7 @@ const char* ts_status_str(ts_status s) {
         case TS_ERR_BAD_INDEX: return "TS_ERR_BAD_INDEX";
         case TS_ERR_TIMEOUT: return "TS_ERR_TIMEOUT";
         case TS_ERR_UNSUPPORTED: return "TS_ERR_UNSUPPORTED";
+        case TS_ERR_SCRATCH: return "TS_ERR_SCRATCH";
     }
     return "TS_ERR_UNKNOWN";
 }
@@ -537,6 +582,7 @@ ts_status ts_stack_forward(ts_ffn* const* layers, int n_layers, float* hres, int
         // a caller's list is in memory before the stack starts; from the
         // second layer on, every kernel before the launch has finished with
         // the first layer's wait, so the list may be read before waiting
+        LayerRange range("ffn stack", l);
         ts_status st = stack_layer(layers[l], next_dense ? layers[l + 1] : nullptr, hres, batch, rows,
                                    rows ? n_active[l] : 0, stream, l > 0);
         if (st != TS_OK) return st;
@@ -557,6 +603,19 @@ ts_status ts_ffn_get_active(ts_ffn* h, cudaStream_t stream, int token, int32_t* 
 ts_status ts_ffn_get_error(ts_ffn* h, cudaStream_t stream) {
     if (!h) return TS_ERR_INVALID_ARG;
     return read_status(h->s.status, stream);
+}
+
+ts_status ts_ffn_check_scratch(ts_ffn* h, cudaStream_t stream) {
+    if (!h) return TS_ERR_INVALID_ARG;
+    return check_arena(h->arena, stream);
+}
+
+ts_status ts_ffn_poke_guard(ts_ffn* h, int i) {
+    if (!h || !h->arena.base || i < 0 || (size_t)i >= h->arena.guards.size()) return TS_ERR_INVALID_ARG;
+    const unsigned char v = (unsigned char)~kGuardByte;
+    return cudaMemcpy(h->arena.base + h->arena.guards[(size_t)i], &v, 1, cudaMemcpyHostToDevice) == cudaSuccess
+               ? TS_OK
+               : TS_ERR_CUDA;
 }
 
 ts_status ts_ffn_set_test_stall(ts_ffn* h, int on) {
@@ -728,6 +787,7 @@ ts_status ts_moe_stack_forward(ts_moe* const* layers, int n_layers, float* hres,
             return TS_ERR_INVALID_ARG;
     }
     for (int l = 0; l < n_layers; ++l) {
+        LayerRange range("moe stack", l);
         ts_status st = moe_layer(layers[l], nullptr, hres, batch, nullptr, stream);
         if (st != TS_OK) return st;
         layers[l]->last_batch = batch;
@@ -782,6 +842,11 @@ ts_status ts_moe_get_error(ts_moe* h, cudaStream_t stream) {
     return read_status(h->s.status, stream);
 }
 
+ts_status ts_moe_check_scratch(ts_moe* h, cudaStream_t stream) {
+    if (!h) return TS_ERR_INVALID_ARG;
+    return check_arena(h->arena, stream);
+}
+
 // ---------------------------------------------------------------------------
 // graphs
 // ---------------------------------------------------------------------------
@@ -830,6 +895,11 @@ void ts_predictor_destroy(ts_predictor* p) {
     if (!p) return;
     if (p->arena.base) cudaFree(p->arena.base);
     delete p;
+}
+
+ts_status ts_predictor_check_scratch(ts_predictor* p, cudaStream_t stream) {
+    if (!p) return TS_ERR_INVALID_ARG;
+    return check_arena(p->arena, stream);
 }
 
 }  // extern "C"
@@ -891,6 +961,7 @@ ts_status ts_stack_forward_predicted(ts_ffn* const* layers, ts_predictor* const*
             remember(h, batch, lists[l], 0);
             continue;
         }
+        LayerRange range("predicted stack", l);
         PredictLaunch q = predict_launch(preds[l], batch, K[l], lists[l], nullptr);
         q.h = hres;
         ts_status st = cuda_status(launch_predict(q, elem_size(preds[l]->dt), stream, true));

@@ -144,7 +144,7 @@ __global__ void __launch_bounds__(kDownWarps * kWarp) k_down(const FfnLaunch a) 
                 if (i < n) {
                     const int2 en = s_list[i];
                     const int e = es.act[en.x];
-                    const int j = a.rows ? a.rows[en.y] : en.y;
+                    const int j = debug_row(a.rows ? a.rows[en.y] : en.y, a.m, a.status);
                     if (col < d)
                         wv[u] = ld_stream(static_cast<const T*>(a.ex[e].wd) + (size_t)j * d + col);
                     const float* cp = a.cval + ((size_t)e * kMaxPass) * a.cval_tok_stride + en.y;

@@ -549,7 +549,7 @@ __device__ void produce(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned char*
             mbar_arrive(&sh.full[slot]);
         } else {
             mbar_arrive_expect_tx(&sh.full[slot], row_bytes);
-            tma_load_1d(ring + (size_t)slot * cfg.slot_bytes, w + (size_t)j * row_elems, row_bytes,
+            tma_load_1d(ring + (size_t)slot * cfg.slot_bytes, w + (size_t)debug_row(j, a.m, a.status) * row_elems, row_bytes,
                         &sh.full[slot]);
         }
         ++issued;
@@ -835,7 +835,8 @@ __device__ void produce_mma(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
             mbar_arrive_expect_tx(&sh.full[g], (unsigned)__popc(mask) * row_bytes);
             for (unsigned m = mask; m; m &= m - 1u) {
                 const int r = __ffs(m) - 1;
-                tma_load_1d(ring + ((size_t)g * kChunk + r) * mc.w_stride, w + (size_t)jr[r] * a.row_bytes, row_bytes,
+                tma_load_1d(ring + ((size_t)g * kChunk + r) * mc.w_stride,
+                            w + (size_t)debug_row(jr[r], a.m, a.status) * a.row_bytes, row_bytes,
                             &sh.full[g]);
             }
         }
@@ -1200,7 +1201,7 @@ __device__ void consume_q4w(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned c
         unsigned char* dst = ring + (size_t)(2 * cidx + slot) * kQ4Rows * mc.w_stride;
         int i = 0;
         for (unsigned m = rows; m; m &= m - 1u, ++i) {
-            const int j = s.jr[__ffs(m) - 1];
+            const int j = debug_row(s.jr[__ffs(m) - 1], a.m, a.status);
             const unsigned char* src = w + (size_t)j * row_bytes;
             unsigned char* drow = dst + (size_t)i * mc.w_stride;
             for (int k = lane; k < row_chunks; k += kWarp) cp_async16(drow + 16 * k, src + 16 * k);
@@ -1626,7 +1627,7 @@ __device__ void consume_rows(const FfnLaunch& a, GateUpShared<NT>& sh, unsigned 
         volatile ChunkState<NT>& s = tab[c];
         const int e = s.e;
         const unsigned char* w = static_cast<const unsigned char*>(kind == kTaskGate ? a.ex[e].wg : a.ex[e].wu);
-        const unsigned char* src = w + (size_t)s.jr[r] * row_bytes;
+        const unsigned char* src = w + (size_t)debug_row(s.jr[r], a.m, a.status) * row_bytes;
         unsigned char* dst = ring + (size_t)(cidx * P + slot) * rc.slot_bytes;
         for (int k = lane; k < row_chunks; k += kWarp) cp_async16(dst + 16 * k, src + 16 * k);
         cp_async_commit();

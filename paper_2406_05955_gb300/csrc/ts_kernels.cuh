@@ -26,6 +26,21 @@ constexpr int kRouterMaxD = 16384;  // router keeps one fp32 activation row in s
 // device status bits (OR-ed into the handle's status word)
 constexpr unsigned kStatusBadIndex = 1u;
 constexpr unsigned kStatusTimeout = 2u;
+
+// Gather-index checks of the debug build (compiled with -DTS_DEBUG): every row
+// index a kernel is about to gather is compared with the row count m; a bad one
+// is recorded as kStatusBadIndex in the status word and replaced by row 0, so
+// the kernel stays in bounds. The release build validates the caller's lists
+// once, where it reads them, and compiles these checks out.
+#ifdef TS_DEBUG
+__device__ __forceinline__ int debug_row(int j, int m, unsigned* status) {
+    if ((unsigned)j < (unsigned)m) return j;
+    atomicOr(status, kStatusBadIndex);
+    return 0;
+}
+#else
+__device__ __forceinline__ int debug_row(int j, int, unsigned*) { return j; }
+#endif
 // Bound on any device-side wait: a wait that lasts longer records
 // kStatusTimeout and the kernel winds down instead of hanging.
 constexpr unsigned long long kWaitLimitNs = 1000000000ull;

@@ -266,7 +266,7 @@ __device__ bool gu_tile_tc(const WideLaunch& L, const __nv_bfloat16* w, const in
         const int r = q >> 3, c = q & 7;
         const int j = rows_j[r];
         wok[i] = j >= 0;
-        wsrc[i] = w + (size_t)(j >= 0 ? j : 0) * d + c * 8;
+        wsrc[i] = w + (size_t)(j >= 0 ? debug_row(j, L.m, L.status) : 0) * d + c * 8;
         wdst[i] = swz(r, c, 128);
     }
     constexpr int kXPer = (C::NP * 8 + kGuThreads - 1) / kGuThreads;
@@ -571,7 +571,7 @@ __global__ void __launch_bounds__(kDownThreads) k_wide_down(const WideLaunch L) 
                 const int r = q >> 5, c = q & 31;
                 const int li = kst * kDownK + r;
                 const int p = li < n_piece ? pos[li] : -1;
-                const int j = p >= 0 ? (L.rows ? L.rows[p] : p) : 0;
+                const int j = debug_row(p >= 0 ? (L.rows ? L.rows[p] : p) : 0, L.m, L.status);
                 cp16(base + r * (kDownCols * 2) + (((c & ~7) | ((c ^ r) & 7)) << 4),
                      L.wd + (size_t)j * d + n0 + c * 8, p >= 0);
             }
@@ -752,7 +752,7 @@ __global__ void __launch_bounds__(kGuThreads) k_wide_down_tc(const WideLaunch L)
             const int r = qq >> 4, c16 = qq & 15;
             const int li = kb * kTcDownK + r;
             const int pp = li < n_list ? pos[li - piece * kTcDownPiece] : -1;
-            const int j = pp >= 0 ? (L.rows ? L.rows[pp] : pp) : 0;
+            const int j = debug_row(pp >= 0 ? (L.rows ? L.rows[pp] : pp) : 0, L.m, L.status);
             const int h = c16 >> 3, c = c16 & 7;
             cp16(base + h * C::kAHalf + swz(r, c, 128), L.wd + (size_t)j * d + n0 + c16 * 8, pp >= 0);
         }

@@ -35,12 +35,30 @@ def test_header_symbols_exported(lib):
     assert set(names) == set(binding.SIGNATURES), "binding signatures and header disagree"
 
 
+def test_debug_library_exports_the_same_symbols(lib):
+    from paper_2406_05955_gb300 import build
+
+    assert os.path.exists(build.DEBUG_LIB), "build() also makes the range-checked debug library"
+    raw = ctypes.CDLL(build.DEBUG_LIB)
+    for n in _declared():
+        assert hasattr(raw, n), f"{n} not exported by the debug library"
+
+
+def test_scratch_checks_reject_null_handles(lib):
+    from paper_2406_05955_gb300.binding import TS_ERR_INVALID_ARG
+
+    assert lib.ts_ffn_check_scratch(None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_moe_check_scratch(None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_predictor_check_scratch(None, None) == TS_ERR_INVALID_ARG
+    assert lib.ts_ffn_poke_guard(None, 0) == TS_ERR_INVALID_ARG
+
+
 def test_status_strings_and_version(lib):
     from paper_2406_05955_gb300 import binding
 
-    names = [binding.status_str(s) for s in range(7)]
+    names = [binding.status_str(s) for s in range(8)]
     assert names == ["TS_OK", "TS_ERR_INVALID_ARG", "TS_ERR_CUDA", "TS_ERR_OOM", "TS_ERR_BAD_INDEX",
-                     "TS_ERR_TIMEOUT", "TS_ERR_UNSUPPORTED"]
+                     "TS_ERR_TIMEOUT", "TS_ERR_UNSUPPORTED", "TS_ERR_SCRATCH"]
     assert binding.status_str(99) == "TS_ERR_UNKNOWN"
     assert lib.ts_version() >= 100
 
