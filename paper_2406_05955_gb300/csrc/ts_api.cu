@@ -451,7 +451,7 @@ ts_status read_status(unsigned* status_dev, cudaStream_t stream) {
 // rows (all, or the list). `next` is the following layer when it runs dense
 // (its first W_gate rows are then prefetched into L2), else nullptr.
 ts_status stack_layer(ts_ffn* h, const ts_ffn* next, float* hres, int batch, const int32_t* rows, int nr,
-                      cudaStream_t stream, bool rows_ready, bool h_ready = false) {
+                      cudaStream_t stream, bool rows_ready, bool h_ready = false, bool trigger_early = false) {
     if (use_wide(h, batch)) {
         WideLaunch L = wide_launch(h, batch, rows, nr);
         L.x = h->w_x;
@@ -469,6 +469,7 @@ ts_status stack_layer(ts_ffn* h, const ts_ffn* next, float* hres, int batch, con
     a.residual_out = 1;
     a.rows_ready = rows != nullptr && rows_ready ? 1 : 0;
     a.h_ready = h_ready ? 1 : 0;
+    a.trigger_early = trigger_early ? 1 : 0;
     if (next != nullptr && batch <= kMaxPass && h->dt != TS_INT4) {
         a.next_wg = next->wg;
         a.next_n_rows = next->m;
@@ -584,7 +585,7 @@ ts_status ts_stack_forward(ts_ffn* const* layers, int n_layers, float* hres, int
         // the first layer's wait, so the list may be read before waiting
         LayerRange range("ffn stack", l);
         ts_status st = stack_layer(layers[l], next_dense ? layers[l + 1] : nullptr, hres, batch, rows,
-                                   rows ? n_active[l] : 0, stream, l > 0);
+                                   rows ? n_active[l] : 0, stream, l > 0, false, l + 1 < n_layers);
         if (st != TS_OK) return st;
     }
     return TS_OK;

@@ -233,8 +233,13 @@ constexpr int kRedBatch = 6;  // partial blocks a half-warp has in flight
 template <int NT>
 __global__ void __launch_bounds__(kRedThreads) k_down_reduce(const FfnLaunch a) {
     __shared__ float4 red[kRedWarps][NT][kRedLanes];
+    // In an FFN stack the next kernel is the next layer's gate+up kernel: it
+    // may be scheduled at once (it waits for this one to finish before it
+    // reads h), and its CTAs take each SM as the gate+up CTA there exits, so
+    // its prologue (launch, list set-up) overlaps this reduction.
+    if (a.trigger_early) pdl_launch_dependents();
     pdl_wait();
-    pdl_launch_dependents();
+    if (!a.trigger_early) pdl_launch_dependents();
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int hw = lane / kRedLanes;

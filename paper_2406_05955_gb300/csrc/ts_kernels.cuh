@@ -110,6 +110,10 @@ struct FfnLaunch {
     // predictor's kernels sit between the last writer of h and this launch),
     // so the activations may be staged before waiting for them.
     int h_ready;
+    // Nonzero when the kernel after this launch's reduction is the next
+    // layer's gate+up kernel (FFN stacks): the reduction lets it be scheduled
+    // before its own wait. (MoE and predicted stacks measured slower so.)
+    int trigger_early;
     // Stack mode: the next layer's W_gate (nullptr: none), its row count and
     // its gate+up grid. The gathered down kernel (passes of 4-8 tokens),
     // before waiting for the gate+up kernel, prefetches into L2 the first
