@@ -967,7 +967,9 @@ ts_status ts_stack_forward_predicted(ts_ffn* const* layers, ts_predictor* const*
         q.h = hres;
         ts_status st = cuda_status(launch_predict(q, elem_size(preds[l]->dt), stream, true));
         // the predictor's three kernels ran after the last writer of h
-        if (st == TS_OK) st = stack_layer(h, nullptr, hres, batch, lists[l], K[l], stream, false, true);
+        // the reduction lets the next layer's predictor kernels be scheduled
+        // before their wait, as it does for the next gate+up kernel
+        if (st == TS_OK) st = stack_layer(h, nullptr, hres, batch, lists[l], K[l], stream, false, true, l + 1 < n_layers);
         if (st != TS_OK) return st;
     }
     return TS_OK;
