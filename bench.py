@@ -56,7 +56,7 @@ NOMINAL_HBM_GBS = 7900.0
 KERNEL_SOURCES = ("paper_2406_05955_gb300/csrc/ts_gate_up.cu", "paper_2406_05955_gb300/csrc/ts_kernels.cuh")
 NCU_TRAFFIC = {"bytes": {"bf16": 164.42e6, "int4": 45.68e6},
                "sources": KERNEL_SOURCES,
-               "sha256": "a804f2637c5f68d9a7858bb3f1236f67397ec9e3f2ab36d31b797236ad620ea2"}
+               "sha256": "6fb244ad1f3a363b7a9054f3a6e3ab5cb12d552ecf90b113a1a7d7db02fb28a1"}
 
 
 def kernel_sources_sha256(paths) -> str:

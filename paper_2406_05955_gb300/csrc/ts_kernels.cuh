@@ -111,8 +111,10 @@ struct FfnLaunch {
     // so the activations may be staged before waiting for them.
     int h_ready;
     // Nonzero when the kernel after this launch's reduction is the next
-    // layer's gate+up kernel (FFN stacks): the reduction lets it be scheduled
-    // before its own wait. (MoE and predicted stacks measured slower so.)
+    // layer's first kernel in an FFN stack (its gate+up kernel, or the
+    // predictor's first kernel): the reduction lets it be scheduled before
+    // its own wait. (The MoE stack, whose router comes next, measured slower
+    // so.)
     int trigger_early;
     // Stack mode: the next layer's W_gate (nullptr: none), its row count and
     // its gate+up grid. The gathered down kernel (passes of 4-8 tokens),
