@@ -523,12 +523,15 @@ ts_status ts_ffn_forward_topk(ts_ffn* h, const void* x, int batch, float* y, cud
     a.x = x;
     a.y = y;
     for (int t0 = 0; t0 < batch; t0 += kMaxPass) {
-        // passes of at least 4 tokens: the down projection runs after the mask
+        // the down projection runs after the mask: passes of 1-2 tokens take
+        // the row kernel without its per-CTA down partial (a null partial
+        // buffer), then the mask, then the gathered down kernel
         const int nt = std::min(kMaxPass, batch - t0);
-        const int w = std::max(4, pow2_tokens(nt));
+        const int w = nt <= kAccMaxTokens ? pow2_tokens(nt) : std::max(4, pow2_tokens(nt));
         a.tok0 = t0;
         a.nt = nt;
         a.bits_tok_base = t0;
+        a.partial = w <= kAccMaxTokens ? nullptr : h->s.partial;
         a.partial_ctas = h->grid[w];
         ts_status st = cuda_status(launch_gate_up(a, h->dt, w, h->grid[w], stream, true));
         if (st == TS_OK) st = cuda_status(launch_topk(a, keep, stream));

@@ -766,9 +766,10 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up(const F
     consume<T, NT>(a, sh, ring, xs, cfg, warp - 1, lane);
     if constexpr (NT <= kAccMaxTokens) {
         // every chunk is finalized and every ring copy consumed once all
-        // consumers are here
+        // consumers are here (no partial buffer: the caller runs the
+        // gathered down kernel after a mask instead)
         named_bar_sync(1, cthreads);
-        down_partial<T, NT>(a, sh, i0, i1, n_chunks, warp - 1, lane);
+        if (a.partial != nullptr) down_partial<T, NT>(a, sh, i0, i1, n_chunks, warp - 1, lane);
     }
 }
 
@@ -1820,7 +1821,8 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(co
         named_bar_sync(1, cthreads);
     };
     consume_rows<T, NT>(a, sh, ring, xs, tab, ulist, rc, i0, i1, n_chunks, warp - 1, lane, stage);
-    down_partial<T, NT>(a, sh, i0, i1, n_chunks, warp - 1, lane);
+    // no partial buffer: the caller runs the gathered down kernel after a mask instead
+    if (a.partial != nullptr) down_partial<T, NT>(a, sh, i0, i1, n_chunks, warp - 1, lane);
 }
 
 // ---------------------------------------------------------------------------
@@ -2066,7 +2068,9 @@ static cudaError_t launch_t(const FfnLaunch& a, int grid, cudaStream_t stream, b
     if (gate_up_config(sizeof(T) == 2 ? 1 : 0, a.d, n_x, g_optin, &cfg.slots, &cfg.slot_bytes,
                        &cfg.xs_stride, &smem) != 0)
         return cudaErrorInvalidValue;
-    if (NT <= kAccMaxTokens && (a.partial == nullptr || a.partial_slots < n_x || a.partial_ctas < grid))
+    // a null partial buffer skips the per-CTA down partial (the caller runs
+    // the gathered down kernel instead); a given one must hold every CTA
+    if (NT <= kAccMaxTokens && a.partial != nullptr && (a.partial_slots < n_x || a.partial_ctas < grid))
         return cudaErrorInvalidValue;
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(grid);
@@ -2123,7 +2127,7 @@ static cudaError_t launch_rows_t(const FfnLaunch& a, int grid, cudaStream_t stre
     const size_t smem = rows_smem((int)sizeof(T), a.d, NT, g_optin - kSmemMargin, &rc);
     if (smem + kSmemMargin > (size_t)g_optin) return cudaErrorInvalidValue;
     const int n_x = a.route ? a.batch : a.nt;
-    if (n_x > NT || a.partial == nullptr || a.partial_slots < n_x || a.partial_ctas < grid)
+    if (n_x > NT || (a.partial != nullptr && (a.partial_slots < n_x || a.partial_ctas < grid)))
         return cudaErrorInvalidValue;
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(grid);

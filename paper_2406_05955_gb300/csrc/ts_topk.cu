@@ -10,6 +10,36 @@ namespace tsffn {
 namespace {
 
 constexpr int kSelThreads = 1024;
+constexpr int kSelWarps = kSelThreads / kWarp;
+
+// Exclusive prefix of v over the block in thread order, and the block total
+// (warp shuffles, then one warp over the warp sums).
+__device__ __forceinline__ int block_excl_scan(int v, int* s_warp, int* s_total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < kWarp; o <<= 1) {
+        const int n = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += n;
+    }
+    if (lane == kWarp - 1) s_warp[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        const int w = lane < kSelWarps ? s_warp[lane] : 0;
+        int wi = w;
+#pragma unroll
+        for (int o = 1; o < kWarp; o <<= 1) {
+            const int n = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += n;
+        }
+        if (lane < kSelWarps) s_warp[lane] = wi - w;
+        if (lane == kWarp - 1) *s_total = wi;
+    }
+    __syncthreads();
+    const int r = s_warp[warp] + incl - v;
+    __syncthreads();  // s_warp is reused by the next scan
+    return r;
+}
 
 // One CTA per token of the pass. c > 0 at a both-active row, so the fp32 bit
 // pattern orders the candidates; an MSB-first radix select (four 8-bit
@@ -18,7 +48,7 @@ constexpr int kSelThreads = 1024;
 // ranges of the bitmap, so a block prefix over the threads is row order.
 __global__ void __launch_bounds__(kSelThreads) k_topk_select(const FfnLaunch a, int keep) {
     __shared__ unsigned hist[256];
-    __shared__ int s_part[kSelThreads];
+    __shared__ int s_warp[kSelWarps];
     __shared__ unsigned s_prefix, s_mask;
     __shared__ int s_remaining, s_total;
     pdl_wait();
@@ -35,12 +65,8 @@ __global__ void __launch_bounds__(kSelThreads) k_topk_select(const FfnLaunch a, 
     // candidates
     int cnt = 0;
     for (int b = b0; b < b1; ++b) cnt += __popc((unsigned)bb[b]);
-    s_part[tid] = cnt;
-    __syncthreads();
+    block_excl_scan(cnt, s_warp, &s_total);
     if (tid == 0) {
-        int t = 0;
-        for (int i = 0; i < kSelThreads; ++i) t += s_part[i];
-        s_total = t;
         s_prefix = 0u;
         s_mask = 0u;
         s_remaining = keep;
@@ -59,17 +85,38 @@ __global__ void __launch_bounds__(kSelThreads) k_topk_select(const FfnLaunch a, 
                 if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
             }
         __syncthreads();
-        if (tid == 0) {
-            // the digit of the keep-th largest key among those with the prefix
-            int remaining = s_remaining;
-            int dg = 255;
-            for (; dg > 0; --dg) {
-                if ((int)hist[dg] >= remaining) break;
-                remaining -= (int)hist[dg];
+        if (tid < kWarp) {
+            // the digit of the keep-th largest key among those with the
+            // prefix: lane l holds digits 255 - 8l .. 248 - 8l, highest first
+            const int lane = tid;
+            const int rem0 = s_remaining;
+            int c8[8], sum = 0;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                c8[q] = (int)hist[255 - 8 * lane - q];
+                sum += c8[q];
             }
-            s_prefix = prefix | ((unsigned)dg << shift);
-            s_mask = mask | (255u << shift);
-            s_remaining = remaining;  // how many keys equal to the final prefix are kept, at the end
+            int incl = sum;
+#pragma unroll
+            for (int o = 1; o < kWarp; o <<= 1) {
+                const int n = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += n;
+            }
+            int above = incl - sum;  // keys in higher digits
+            // the highest digit whose count from the top reaches rem0 (digit
+            // 0 when none does, as a scan from the top stops at the bottom)
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int dg = 255 - 8 * lane - q;
+                const bool reach = above + c8[q] >= rem0;
+                const bool first = dg == 255 || above < rem0;
+                if (first && (reach || dg == 0)) {
+                    s_prefix = prefix | ((unsigned)dg << shift);
+                    s_remaining = rem0 - above;  // how many keys equal to the final prefix are kept, at the end
+                }
+                above += c8[q];
+            }
+            if (lane == 0) s_mask = mask | (255u << shift);
         }
         __syncthreads();
     }
@@ -79,18 +126,7 @@ __global__ void __launch_bounds__(kSelThreads) k_topk_select(const FfnLaunch a, 
     int eq = 0;
     for (int b = b0; b < b1; ++b)
         for (unsigned bits = bb[b]; bits; bits &= bits - 1u) eq += key_of(b * 8 + __ffs(bits) - 1) == T;
-    s_part[tid] = eq;
-    __syncthreads();
-    if (tid == 0) {
-        int run = 0;
-        for (int i = 0; i < kSelThreads; ++i) {
-            const int v = s_part[i];
-            s_part[i] = run;
-            run += v;
-        }
-    }
-    __syncthreads();
-    int rank = s_part[tid];
+    int rank = block_excl_scan(eq, s_warp, &s_total);
     for (int b = b0; b < b1; ++b) {
         unsigned kept = 0u;
         for (unsigned bits = bb[b]; bits; bits &= bits - 1u) {
