@@ -114,6 +114,18 @@ __device__ __forceinline__ int xs_index(int i) {
     return i;
 }
 
+// Writes staged activations into an fp32 row at xs_index positions: one
+// element, or four consecutive ones (i a multiple of 4, which xs_index keeps
+// contiguous and 16-byte aligned) in one store.
+template <typename T>
+struct XsPut {
+    float* row;
+    __device__ __forceinline__ void operator()(int i, float v) const { row[xs_index<T>(i)] = v; }
+    __device__ __forceinline__ void operator()(int i, float4 v) const {
+        *reinterpret_cast<float4*>(row + xs_index<T>(i)) = v;
+    }
+};
+
 // acc[k] = sum_i row[i] * x_{xt[k]}[i] for k < ntok (row in shared memory).
 // Each lane keeps ACC independent partial sums per token (element q of a
 // 16-byte vector goes to sum q % ACC) so the FMAs do not form one serial
@@ -760,7 +772,7 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up(const F
         float* xrow = xs + (size_t)t * cfg.xs_stride;
         stage_act_row<T>(a.norm_from_h ? a.h + (size_t)(x_tok0 + t) * a.d : nullptr,
                          static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d, a.d, ctid, cthreads, sh.red,
-                         [&](int i, float v) { xrow[xs_index<T>(i)] = v; });
+                         XsPut<T>{xrow});
     }
     named_bar_sync(1, cthreads);
     consume<T, NT>(a, sh, ring, xs, cfg, warp - 1, lane);
@@ -1782,7 +1794,7 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(co
         for (int t = 0; t < n_x; ++t) {
             float* xrow = xs + (size_t)t * rc.xs_stride;
             stage_act_row<T>(a.h + (size_t)(x_tok0 + t) * a.d, nullptr, a.d, ctid, cthreads, sh.red,
-                             [&](int i, float v) { xrow[xs_index<T>(i)] = v; });
+                             XsPut<T>{xrow});
         }
         named_bar_sync(1, cthreads);
         pdl_wait();
@@ -1815,7 +1827,7 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_gate_up_rows(co
             float* xrow = xs + (size_t)t * rc.xs_stride;
             stage_act_row<T>(a.norm_from_h ? a.h + (size_t)(x_tok0 + t) * a.d : nullptr,
                              static_cast<const T*>(a.x) + (size_t)(x_tok0 + t) * a.d, a.d, ctid, cthreads, sh.red,
-                             [&](int i, float v) { xrow[xs_index<T>(i)] = v; }, once);
+                             XsPut<T>{xrow}, once);
         }
         once();
         named_bar_sync(1, cthreads);
@@ -2007,7 +2019,7 @@ __global__ void __launch_bounds__(GateUpWarps<NT>::THREADS, 1) k_stack_rows(cons
             for (int t = 0; t < la.nt; ++t) {
                 float* xrow = xs + (size_t)t * rc.xs_stride;
                 stage_act_row<T>(S.h + (size_t)t * la.d, nullptr, la.d, ctid, cthreads, sh.red,
-                                 [&](int i, float v) { xrow[xs_index<T>(i)] = v; }, once);
+                                 XsPut<T>{xrow}, once);
             }
             once();
             named_bar_sync(1, cthreads);

@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <type_traits>
+
 namespace tsffn {
 
 constexpr int kWarp = 32;
@@ -416,10 +418,16 @@ __device__ __forceinline__ void stage_act_row(const float* __restrict__ h, const
                 const int q = g0 + ctid + k * cthreads;
                 if (q < d4) {
                     const float4 w = kept ? v[k] : __ldcg(reinterpret_cast<const float4*>(h + 4 * (size_t)q));
-                    put(4 * q, norm(4 * q, w.x));
-                    put(4 * q + 1, norm(4 * q + 1, w.y));
-                    put(4 * q + 2, norm(4 * q + 2, w.z));
-                    put(4 * q + 3, norm(4 * q + 3, w.w));
+                    if constexpr (std::is_invocable_v<Put, int, float4>) {
+                        // elements 4q .. 4q + 3 in one store
+                        put(4 * q, make_float4(norm(4 * q, w.x), norm(4 * q + 1, w.y), norm(4 * q + 2, w.z),
+                                               norm(4 * q + 3, w.w)));
+                    } else {
+                        put(4 * q, norm(4 * q, w.x));
+                        put(4 * q + 1, norm(4 * q + 1, w.y));
+                        put(4 * q + 2, norm(4 * q + 2, w.z));
+                        put(4 * q + 3, norm(4 * q + 3, w.w));
+                    }
                 }
             }
         }
