@@ -11,6 +11,7 @@ namespace {
 
 constexpr int kSelThreads = 1024;
 constexpr int kSelWarps = kSelThreads / kWarp;
+constexpr int kKeyCache = 8;  // candidate keys a thread keeps in shared memory (the rest are re-read)
 
 // Exclusive prefix of v over the block in thread order, and the block total
 // (warp shuffles, then one warp over the warp sums).
@@ -45,9 +46,12 @@ __device__ __forceinline__ int block_excl_scan(int v, int* s_warp, int* s_total)
 // pattern orders the candidates; an MSB-first radix select (four 8-bit
 // digits) finds the keep-th largest key T, then the rows with key > T and the
 // first rows (ascending) with key == T are kept. Threads own contiguous byte
-// ranges of the bitmap, so a block prefix over the threads is row order.
+// ranges of the bitmap, so a block prefix over the threads is row order; each
+// thread keeps its first kKeyCache candidate keys in shared memory for the
+// passes.
 __global__ void __launch_bounds__(kSelThreads) k_topk_select(const FfnLaunch a, int keep) {
     __shared__ unsigned hist[256];
+    __shared__ unsigned s_key[kKeyCache * kSelThreads];  // [slot][thread]: a thread's first candidates
     __shared__ int s_warp[kSelWarps];
     __shared__ unsigned s_prefix, s_mask;
     __shared__ int s_remaining, s_total;
@@ -60,11 +64,16 @@ __global__ void __launch_bounds__(kSelThreads) k_topk_select(const FfnLaunch a, 
     const int n_bytes = (a.n_rows + 7) / 8;
     const int per = (n_bytes + kSelThreads - 1) / kSelThreads;
     const int b0 = min(tid * per, n_bytes), b1 = min(b0 + per, n_bytes);
-    auto key_of = [&](int p) { return __float_as_uint(cv[p]); };
+    auto key_ld = [&](int p) { return __float_as_uint(cv[p]); };
+    // the i-th candidate of this thread (row p): from shared memory for the
+    // first kKeyCache, else from c
+    auto key_of = [&](int i, int p) { return i < kKeyCache ? s_key[i * kSelThreads + tid] : key_ld(p); };
 
-    // candidates
+    // candidates, the first kKeyCache keys of each thread kept in shared memory
     int cnt = 0;
-    for (int b = b0; b < b1; ++b) cnt += __popc((unsigned)bb[b]);
+    for (int b = b0; b < b1; ++b)
+        for (unsigned bits = bb[b]; bits; bits &= bits - 1u, ++cnt)
+            if (cnt < kKeyCache) s_key[cnt * kSelThreads + tid] = key_ld(b * 8 + __ffs(bits) - 1);
     block_excl_scan(cnt, s_warp, &s_total);
     if (tid == 0) {
         s_prefix = 0u;
@@ -78,10 +87,10 @@ __global__ void __launch_bounds__(kSelThreads) k_topk_select(const FfnLaunch a, 
         for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
         __syncthreads();
         const unsigned prefix = s_prefix, mask = s_mask;
+        int i = 0;
         for (int b = b0; b < b1; ++b)
-            for (unsigned bits = bb[b]; bits; bits &= bits - 1u) {
-                const int p = b * 8 + __ffs(bits) - 1;
-                const unsigned key = key_of(p);
+            for (unsigned bits = bb[b]; bits; bits &= bits - 1u, ++i) {
+                const unsigned key = key_of(i, b * 8 + __ffs(bits) - 1);
                 if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
             }
         __syncthreads();
@@ -124,15 +133,19 @@ __global__ void __launch_bounds__(kSelThreads) k_topk_select(const FfnLaunch a, 
     const int need_eq = s_remaining;
     // rank of each key == T in row order
     int eq = 0;
-    for (int b = b0; b < b1; ++b)
-        for (unsigned bits = bb[b]; bits; bits &= bits - 1u) eq += key_of(b * 8 + __ffs(bits) - 1) == T;
+    {
+        int i = 0;
+        for (int b = b0; b < b1; ++b)
+            for (unsigned bits = bb[b]; bits; bits &= bits - 1u, ++i) eq += key_of(i, b * 8 + __ffs(bits) - 1) == T;
+    }
     int rank = block_excl_scan(eq, s_warp, &s_total);
+    int i = 0;
     for (int b = b0; b < b1; ++b) {
         unsigned kept = 0u;
-        for (unsigned bits = bb[b]; bits; bits &= bits - 1u) {
+        for (unsigned bits = bb[b]; bits; bits &= bits - 1u, ++i) {
             const int r = __ffs(bits) - 1;
             const int p = b * 8 + r;
-            const unsigned key = key_of(p);
+            const unsigned key = key_of(i, p);
             bool keep_it = key > T;
             if (key == T) keep_it = rank++ < need_eq;
             if (keep_it)
