@@ -56,7 +56,7 @@ NOMINAL_HBM_GBS = 7900.0
 KERNEL_SOURCES = ("paper_2406_05955_gb300/csrc/ts_gate_up.cu", "paper_2406_05955_gb300/csrc/ts_kernels.cuh")
 NCU_TRAFFIC = {"bytes": {"bf16": 164.46e6, "int4": 45.69e6},
                "sources": KERNEL_SOURCES,
-               "sha256": "36e23ba3ed72ecb1a6629157eafbf0f2015433c7dce996390ef50e066be91cdf"}
+               "sha256": "1dffd86c23421f56c66f947e8e8ada4f087e60ca9d85d582a0f1422c09050c43"}
 
 
 def kernel_sources_sha256(paths) -> str:

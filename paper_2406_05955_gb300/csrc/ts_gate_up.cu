@@ -1,34 +1,32 @@
 // ts_gate_up.cu -- fused gate GEMV + ReLU + compaction and gathered up
-// projection + dReLU product + second compaction (Eq. 1 with Eq. 2).
-//
-// Persistent kernel, one CTA per SM: a producer warp and C consumer
-// warps around a ring of S whole-row slots in shared memory.
-//   * Work item = (expert, chunk of kChunk consecutive rows of the row space);
-//     each CTA owns a contiguous range of items.
-//   * A task is one row in one slot. The producer thread fills free slots
-//     with 1-D bulk copies (cp.async.bulk, 8 KB per row at d=4096 bf16)
-//     completing on the slot's "full" mbarrier. Order: the gate rows of chunk
-//     c, then the up rows of chunk c-kLookahead -- those whose gate
-//     pre-activation is positive for some token, known once that chunk's gate
-//     rows are done. So W_up bytes are read only for gate-active neurons while
-//     the ring stays full.
-//   * Consumer warps take tasks round-robin, dot the slot's row with the
-//     activations (fp32 in shared memory, permuted so 16-byte reads are
-//     conflict-free), release the slot, and record g or u in the chunk's
-//     window state. Each consumer owns two or more slots, so one is in
-//     flight while its owner computes on another. The warp that completes a
-//     chunk's gate rows publishes its gate-active mask to the producer; the warp that completes its up rows
-//     writes the chunk's per-token bitmap bytes, union bytes and
-//     c = w_route * g * u, then frees the window slot.
-//   * In detected mode for a single FFN the producer needs nothing from earlier
-//     kernels, so it starts streaming W_gate before griddepcontrol.wait; the
-//     consumers wait before reading the activations.
-//   * Passes of up to kAccMaxTokens tokens also do this CTA's share of the
-//     down projection at the end (down_partial): the CTA's W_down rows are
-//     read from L2 and summed into its block of the partial
-//     buffer, which the down kernel's reduction adds up over the CTAs.
-// Every mbarrier wait is bounded (kWaitLimitNs); on expiry the status word
-// gets kStatusTimeout and the CTA drains its copies and returns.
+// projection + dReLU product + second compaction (Eq. 1 with Eq. 2), for
+// passes of up to 8 tokens. Every kernel is persistent, one CTA per SM, and
+// works on items = (expert, chunk of kChunk consecutive rows of the row
+// space), each CTA a contiguous range of items; W_up rows are read only for
+// gate-active neurons, and each finished chunk's per-token bitmap bytes,
+// union bytes and c = w_route * g * u are written out (finalize_chunks).
+//   * k_gate_up_rows (bf16, 1-2 tokens, the decode path): no producer. Each
+//     consumer warp copies its own rows with 16-byte cp.async into its own
+//     ring slots, a few rows ahead of the one it computes; a round of chunks
+//     is a gate phase (every gate row shared out one at a time), then an up
+//     phase (every gate-active row), then the chunks are finalised; then the
+//     CTA sums its both-active W_down rows into its block of the partial
+//     buffer (down_partial), which k_down_reduce adds up over the CTAs.
+//   * k_gate_up_q4w (INT4 rows, 1-2 tokens): the same rounds in subtasks of
+//     4 rows, unpacked to bf16 in registers for mma.sync.
+//   * k_gate_up_mma (bf16, 4-8 tokens): a producer thread fills a ring of
+//     8-row groups with 1-D bulk copies; all consumer warps share each group
+//     over K slices with mma.sync.
+//   * k_gate_up (fp32, and bf16 where the others do not fit): a producer
+//     thread fills a ring of whole-row slots, gate rows of chunk c then the
+//     up rows of chunk c - kLookahead; consumers take slots round-robin.
+//   * k_stack_rows: every layer of a batch-1-2 stack in one cooperative
+//     launch, k_gate_up_rows's phases per layer with grid barriers around
+//     the cross-CTA reduction.
+// Where a kernel's rows do not depend on earlier kernels, it starts copying
+// them before griddepcontrol.wait. Every wait on an mbarrier, a flag or the
+// grid is bounded (kWaitLimitNs); on expiry the status word gets
+// kStatusTimeout and the CTA drains its copies and returns.
 #include <type_traits>
 
 #include "ts_kernels.cuh"
