@@ -114,7 +114,9 @@ ts_status ts_ffn_forward(ts_ffn* h, const void* x, int batch, float* y, cudaStre
  * winning a tie; the others contribute 0.
  *   x, batch, y, stream   as ts_ffn_forward (no predictor list)
  *   keep                  0 <= keep <= m; keep >= the number of dReLU-active
- *                         neurons gives exactly ts_ffn_forward's result
+ *                         neurons gives ts_ffn_forward's result up to the
+ *                         fp32 summation order of the down projection (the
+ *                         masked path gathers W_down by column slices)
  * The per-token both-active sets that ts_ffn_get_active reports afterwards
  * are the kept active neurons. The selection compares the fp32 c values.
  * Errors: TS_ERR_INVALID_ARG for a bad keep or batch, TS_ERR_UNSUPPORTED for
