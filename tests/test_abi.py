@@ -111,3 +111,16 @@ def test_binding_refuses_cpu_tensors():
     w = torch.zeros(8, 64, dtype=torch.bfloat16)
     with pytest.raises(TypeError):
         ts.Ffn(w, w, w)
+
+
+def test_debug_environment_selects_the_debug_library(lib):
+    """TS_FFN_DEBUG=1 makes the binding load libtsffn_debug.so (checked in a child process)."""
+    import subprocess
+    import sys
+
+    code = ("import sys; sys.path.insert(0, %r); from paper_2406_05955_gb300 import binding; "
+            "binding.lib(); print(binding.LIB_PATH)") % ROOT
+    env = dict(os.environ, TS_FFN_DEBUG="1")
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    assert r.stdout.strip().endswith(os.path.join("debug", "libtsffn_debug.so"))
